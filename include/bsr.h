@@ -1,0 +1,153 @@
+/*
+ * bsr.h -- C ABI of the GB300 (sm_103a) block-sparse-row x dense product.
+ *
+ * Section 2.2 of "Algorithm to Compilation Co-design: An Integrated View of
+ * Neural Network Sparsity" (Guo and Huang, 2021) stores a pruned weight
+ * W[M, K] in Block Sparse Row form -- block values, block column indices and
+ * block-row pointers, following SciPy -- and multiplies only the kept blocks
+ * with the input tensor. Eq. 3 partitions W into blocks; here a block is
+ * R x C: R consecutive rows of W (output features) by C consecutive columns
+ * (input features). MB = M/R block rows, KB = K/C block columns.
+ *
+ *   indptr[MB+1]     int32, indptr[0] = 0, non-decreasing, indptr[MB] = nnzb
+ *   indices[nnzb]    int32 block-column index, strictly ascending inside a row
+ *   data[nnzb][R][C] block values, row-major inside each block
+ *
+ * The product (the paper's linear/attention projection, Y = X W^T + b):
+ *   Y[n, i*R + r] = bias[i*R + r]
+ *                 + sum_{p = indptr[i]}^{indptr[i+1]-1} sum_{c<C} X[n, indices[p]*C + c] * data[p][r][c]
+ * with X[N, K] and Y[N, M] row-major. Element types: BSR_F32 (fp32 data, X
+ * and Y, fp32 accumulation, no TF32) or BSR_BF16 (bf16 data, X and Y, fp32
+ * accumulation, Y rounded to nearest even). bias is always fp32 or NULL.
+ *
+ * Conventions.
+ *  - Every call returns a status; the library never aborts, prints or traps.
+ *  - Pointers marked "device" are global-memory pointers of the device that
+ *    was current when the handle was created (for bsr_from_dense: the
+ *    current device).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *    stream). Work is enqueued on it; calls say when they synchronise.
+ *  - Supported shapes: 1 <= R, C and R*C <= 4096, M % R == 0, K % C == 0,
+ *    MB + 1, KB and nnzb below 2^31.
+ *  - One handle must not run bsr_spmm on two streams at once (the split-row
+ *    workspace and staging buffers belong to the handle).
+ */
+#ifndef BSR_H
+#define BSR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    BSR_OK = 0,
+    BSR_ERR_INVALID_ARG = 1, /* NULL where a pointer is needed, negative size, aliasing, bad threshold */
+    BSR_ERR_SHAPE = 2,       /* M % R or K % C non-zero, sizes beyond int32 indexing */
+    BSR_ERR_UNSUPPORTED = 3, /* block shape or dtype not supported */
+    BSR_ERR_CAPACITY = 4,    /* output arrays of bsr_from_dense too small */
+    BSR_ERR_STRUCTURE = 5,   /* indptr/indices are not a canonical BSR structure */
+    BSR_ERR_ALIGNMENT = 6,   /* X or Y not 16-byte aligned, bias not 4-byte aligned */
+    BSR_ERR_CUDA = 7,        /* a CUDA runtime call or kernel launch failed */
+    BSR_ERR_TIMEOUT = 8,     /* a bounded device-side wait gave up (reported by bsr_check_device_status) */
+    BSR_ERR_ALLOC = 9        /* device or host allocation failed */
+} bsr_status_t;
+
+typedef enum { BSR_F32 = 0, BSR_BF16 = 1 } bsr_dtype_t;
+
+typedef struct bsr_handle_s *bsr_handle_t;
+
+/*
+ * bsr_from_dense -- build the BSR arrays of a dense weight on the GPU
+ * (Section 2.2: "data values, indices, and indptr").
+ *
+ * W        device, [M, K] row-major, element type dt.
+ * R, C     block shape. threshold: a block is kept iff at least one element
+ *          w has !(|w| <= threshold) in fp32 (so NaN keeps its block, -0.0
+ *          never does). threshold must be >= 0 and not NaN.
+ * indptr   device, MB+1 int32, always written on success and on CAPACITY.
+ * indices  device, capacity_blocks int32; data: device, capacity_blocks*R*C
+ *          elements. Kept blocks appear in ascending column order per row,
+ *          their values copied bit for bit (sub-threshold values included).
+ * Query:   indices == NULL, data == NULL, capacity_blocks == 0 -> BSR_OK,
+ *          *nnzb_out = number of kept blocks, only indptr written.
+ * If capacity_blocks < nnzb: BSR_ERR_CAPACITY, *nnzb_out set, indices/data
+ *          untouched. nnzb_out (host) may be NULL.
+ * Synchronises `stream` once (to read nnzb). Temporary device memory is
+ * allocated and freed inside the call.
+ */
+bsr_status_t bsr_from_dense(const void *W, int64_t M, int64_t K, int R, int C, float threshold,
+                            bsr_dtype_t dt, int32_t *indptr, int32_t *indices, void *data,
+                            int64_t capacity_blocks, int64_t *nnzb_out, void *stream);
+
+/*
+ * bsr_create -- analyse a BSR structure and build its execution schedule
+ * (the counterpart of the paper's task buffer and auto-scheduler, Section
+ * 2.2: tasks with identical structure are reused).
+ *
+ * indptr, indices, data: device arrays as described above. They are
+ * BORROWED: the caller keeps them alive and unmodified until bsr_destroy.
+ * Validates the structure on the host (one device-to-host copy of indptr and
+ * indices, synchronous): indptr[0] == 0, non-decreasing, indices strictly
+ * ascending per row and < K/C; otherwise BSR_ERR_STRUCTURE.
+ * Owns: the schedule (shared with other handles of identical structure),
+ * the work list, a repacked copy of data in the kernels' layout, a device
+ * status word and workspaces. *out receives the handle.
+ */
+bsr_status_t bsr_create(const int32_t *indptr, const int32_t *indices, const void *data, int R,
+                        int C, int64_t M, int64_t K, bsr_dtype_t dt, bsr_handle_t *out);
+
+/*
+ * bsr_reserve -- size the handle's workspaces for up to N_max tokens so that
+ * later bsr_spmm calls with N <= N_max allocate nothing (needed before
+ * capturing bsr_spmm in a CUDA graph). Synchronous.
+ */
+bsr_status_t bsr_reserve(bsr_handle_t h, int64_t N_max);
+
+/*
+ * bsr_spmm -- Y[N, M] = X[N, K] W^T + bias[M] over the kept blocks.
+ *
+ * X, Y     row-major, element type of the handle, 16-byte aligned, not
+ *          overlapping (else BSR_ERR_ALIGNMENT / BSR_ERR_INVALID_ARG).
+ *          Both device pointers, or both host pointers: with host pointers
+ *          the call copies X in and Y out on `stream` through device staging
+ *          buffers owned by the handle; Y is valid once `stream` has
+ *          synchronised.
+ * bias     device, fp32 [M], or NULL for zero.
+ * N        tokens; N == 0 is a no-op returning BSR_OK.
+ * Asynchronous on `stream`; never synchronises unless a workspace must grow
+ * beyond what bsr_reserve sized (then it allocates). Kernel launch failures
+ * return BSR_ERR_CUDA.
+ */
+bsr_status_t bsr_spmm(bsr_handle_t h, const void *X, const float *bias, void *Y, int64_t N,
+                      void *stream);
+
+/*
+ * bsr_check_device_status -- synchronise the device and return the first
+ * error a kernel of this handle recorded (BSR_ERR_TIMEOUT when a bounded
+ * wait gave up, BSR_ERR_STRUCTURE when a kernel met an out-of-range index),
+ * then clear it. BSR_OK if none.
+ */
+bsr_status_t bsr_check_device_status(bsr_handle_t h);
+
+/*
+ * bsr_get_schedule -- a text description of the handle's schedule: kernel
+ * variant, tile sizes, work items, split rows, launches per call and the
+ * schedule-cache statistics, as "key=value" lines. Writes at most len bytes
+ * including the terminating NUL into buf (truncating). Returns
+ * BSR_ERR_INVALID_ARG for a NULL handle or buffer.
+ */
+bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len);
+
+/* bsr_destroy -- release what the handle owns (not the borrowed arrays). NULL is a no-op. */
+void bsr_destroy(bsr_handle_t h);
+
+/* bsr_status_str -- a static, human-readable name for a status code. */
+const char *bsr_status_str(bsr_status_t s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* BSR_H */

@@ -1,0 +1,117 @@
+// Internal declarations shared by the host runtime (api.cpp) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cstdint>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "bsr.h"
+
+namespace bsr {
+
+// One unit of work: block row `row`, stored blocks [p0, p1). slot < 0 writes
+// Y (+ bias) directly; slot >= 0 writes an fp32 partial tile to the workspace
+// at [slot][N][R] and a reduce pass sums the slots of the row.
+struct Item {
+    int32_t row, p0, p1, slot;
+};
+
+// A block row split into pieces: slots [slot0, slot0 + nslot) in piece order.
+struct Split {
+    int32_t row, slot0, nslot, pad;
+};
+
+enum Variant : int {
+    V_GENERIC = 0,   // any R x C, any dtype: one thread per output, global loads
+    V_XSTAGE = 1,    // SIMT, X token tile staged in shared memory, register tiles
+    V_TC = 2,        // tcgen05 tensor cores, bf16 square blocks
+};
+
+const char *variant_name(int v);
+
+// Device-side status word values (first error wins).
+enum : int { DEV_OK = 0, DEV_TIMEOUT = 1, DEV_BAD_INDEX = 2 };
+
+// Everything derived from (device, dtype, R, C, M, K, indptr, indices): shared
+// between handles whose structure is identical.
+struct Schedule {
+    int device = 0;
+    bsr_dtype_t dt = BSR_F32;
+    int R = 1, C = 1;
+    int64_t M = 0, K = 0, MB = 0, KB = 0, nnzb = 0;
+    std::vector<int32_t> indptr, indices;   // host copies (the key)
+    uint64_t hash = 0;
+
+    int variant = V_GENERIC;
+    int tn = 0;            // tokens per CTA
+    int threads = 256;     // threads per CTA
+    int split_len = 0;     // max blocks per item (0: no splitting)
+    int groups = 1;        // item groups per token tile
+    size_t smem = 0;       // dynamic shared memory per CTA
+    std::vector<Item> items;
+    std::vector<Split> splits;
+    std::vector<int32_t> group_begin;   // groups + 1 offsets into items
+    int n_slots = 0;
+    int64_t empty_rows = 0, max_row = 0;
+
+    Item *d_items = nullptr;
+    Split *d_splits = nullptr;
+    int32_t *d_group_begin = nullptr;
+    int32_t *d_indptr = nullptr;        // owned copies of the structure
+    int32_t *d_indices = nullptr;
+
+    std::atomic<int64_t> reuse_count{0};
+    ~Schedule();
+};
+
+struct Handle {
+    int device = 0;
+    bsr_dtype_t dt = BSR_F32;
+    int R = 1, C = 1;
+    int64_t M = 0, K = 0;
+    const void *data = nullptr;         // borrowed
+    void *data_packed = nullptr;        // owned, kernel layout
+    std::shared_ptr<Schedule> sched;
+    int *d_status = nullptr;
+    float *ws = nullptr;                // split-row partials
+    size_t ws_bytes = 0;
+    void *stage_x = nullptr, *stage_y = nullptr;   // for host X / Y
+    size_t stage_x_bytes = 0, stage_y_bytes = 0;
+    bool cache_hit = false;
+};
+
+inline size_t dtype_size(bsr_dtype_t dt) { return dt == BSR_F32 ? 4 : 2; }
+
+// ---- builder (builder.cu)
+cudaError_t launch_builder_count(const void *W, bsr_dtype_t dt, int64_t M, int64_t K, int R, int C,
+                                 float thr, uint8_t *flags, int32_t *counts, int32_t *indptr,
+                                 cudaStream_t s);
+cudaError_t launch_builder_compact(const void *W, bsr_dtype_t dt, int64_t M, int64_t K, int R, int C,
+                                   const uint8_t *flags, const int32_t *indptr, int32_t *indices,
+                                   void *data, cudaStream_t s);
+
+// ---- SpMM kernels (spmm_*.cu)
+struct LaunchArgs {
+    const Schedule *sc;
+    const void *data;      // kernel-layout block values
+    const void *X;
+    const float *bias;
+    void *Y;
+    float *ws;
+    int *status;
+    int64_t N;
+    cudaStream_t stream;
+};
+cudaError_t launch_generic(const LaunchArgs &a);
+cudaError_t launch_reduce(const LaunchArgs &a);
+int launches_per_call(const Schedule &sc);
+
+}  // namespace bsr
+
+// The opaque handle of the C ABI.
+struct bsr_handle_s : public bsr::Handle {};

@@ -1,0 +1,19 @@
+// Schedule construction (work list, split rows, kernel choice) and dispatch.
+#pragma once
+
+#include "bsr_internal.h"
+
+namespace bsr {
+
+// Fills the plan of a Schedule whose key fields (device, dtype, R, C, M, K,
+// indptr, indices) are set, and uploads its device arrays.
+bsr_status_t build_schedule(Schedule &sc);
+
+// Makes the handle's kernel-layout copy of the block values, if the chosen
+// kernel wants one (else the borrowed array is used directly).
+bsr_status_t pack_data(Handle &h);
+
+// Launches every kernel of one bsr_spmm call on a.stream.
+cudaError_t launch_spmm(const LaunchArgs &a);
+
+}  // namespace bsr

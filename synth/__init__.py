@@ -301,7 +301,8 @@ def sweep_sparsities(n_weights: int, config: int = 3) -> List[int]:
 
 
 def config(k: int, dtype: Optional[str] = None, shape: Optional[tuple] = None,
-           n_weights: Optional[int] = None, N: Optional[int] = None) -> Workload:
+           n_weights: Optional[int] = None, N: Optional[int] = None,
+           only: Optional[List[int]] = None) -> Workload:
     """The five benchmark workloads (1-based ``k``), optionally cut down.
 
     1: one 768x768 fp32 weight, 32x1 blocks, 90%; X 128x768.
@@ -312,6 +313,8 @@ def config(k: int, dtype: Optional[str] = None, shape: Optional[tuple] = None,
        X 16384x1024, fp32 or bf16.
     5: one 4096x4096 bf16 weight at 95% with Zipf(1.2) rows, 32x1 or 16x16;
        X 8192x4096 bf16.
+
+    ``only`` keeps just the listed weight indices of workloads 3 and 4.
     """
     if k == 1:
         s = config_seed(1)
@@ -327,16 +330,18 @@ def config(k: int, dtype: Optional[str] = None, shape: Optional[tuple] = None,
     if k == 3:
         nw = 48 if n_weights is None else n_weights
         sp = sweep_sparsities(48)
+        ids = range(nw) if only is None else only
         ws = [make_weight(f"cfg3_L{i // 4}_{'QKVO'[i % 4]}", config_seed(3, i), 768, 768, 32, 1, "f32", sp[i])
-              for i in range(nw)]
+              for i in ids]
         return Workload("cfg3", N or 1024, 768, "f32", ws, seed=config_seed(3))
     if k == 4:
         dt = dtype or "f32"
         R, C = shape or (32, 1)
         si = 0 if (R, C) == (32, 1) else 1
         nw = 96 if n_weights is None else n_weights
+        ids = range(nw) if only is None else only
         ws = [make_weight(f"cfg4_L{i // 4}_{'QKVO'[i % 4]}_{R}x{C}", config_seed(4, i, si), 1024, 1024, R, C, dt, 90)
-              for i in range(nw)]
+              for i in ids]
         return Workload(f"cfg4_{dt}", N or 16384, 1024, dt, ws, seed=config_seed(4, 0, 9))
     if k == 5:
         R, C = shape or (32, 1)
