@@ -10,6 +10,7 @@
 #include <cinttypes>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <unordered_map>
@@ -116,6 +117,7 @@ Schedule::~Schedule() {
     cudaFree(d_splits);
     cudaFree(d_group_begin);
     cudaFree(d_indptr);
+    cudaFree(d_xs_cb);
     cudaFree(d_indices);
 }
 
@@ -236,6 +238,8 @@ bsr_status_t bsr_create(const int32_t *indptr, const int32_t *indices, const voi
     h->M = M;
     h->K = K;
     h->data = data;
+    if (const char *w = getenv("BSR_WAIT_LIMIT_NS")) h->wait_ns = strtoull(w, nullptr, 10);
+    if (const char *w = getenv("BSR_TEST_STALL_CHUNK")) h->stall_chunk = atoi(w);
 
     uint64_t hash = structure_hash(device, dt, R, C, M, K, hp, hi);
     {
@@ -340,7 +344,8 @@ bsr_status_t bsr_spmm(bsr_handle_t h, const void *X, const float *bias, void *Y,
         Xd = h->stage_x;
         Yd = h->stage_y;
     }
-    LaunchArgs a{&sc, h->data_packed ? h->data_packed : h->data, Xd, bias, Yd, h->ws, h->d_status, N, s};
+    LaunchArgs a{&sc, h->data_packed ? h->data_packed : h->data, Xd, bias, Yd, h->ws, h->d_status, N, s,
+                 h->wait_ns, h->stall_chunk};
     if (launch_spmm(a) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_CUDA;

@@ -11,6 +11,7 @@
 #include <vector>
 
 #include "bsr.h"
+#include "xstage.h"
 
 namespace bsr {
 
@@ -56,12 +57,16 @@ struct Schedule {
     std::vector<Item> items;
     std::vector<Split> splits;
     std::vector<int32_t> group_begin;   // groups + 1 offsets into items
+    XsPlan xs;                          // xstage task footprints
     int n_slots = 0;
     int64_t empty_rows = 0, max_row = 0;
+    int sm_count = 148;
 
     Item *d_items = nullptr;
     Split *d_splits = nullptr;
     int32_t *d_group_begin = nullptr;
+    std::vector<int32_t> xs_cb;         // xstage: per item, first block of each K chunk
+    int32_t *d_xs_cb = nullptr;
     int32_t *d_indptr = nullptr;        // owned copies of the structure
     int32_t *d_indices = nullptr;
 
@@ -83,6 +88,8 @@ struct Handle {
     void *stage_x = nullptr, *stage_y = nullptr;   // for host X / Y
     size_t stage_x_bytes = 0, stage_y_bytes = 0;
     bool cache_hit = false;
+    uint64_t wait_ns = 1000000000ull;   // device wait bound (BSR_WAIT_LIMIT_NS at create)
+    int stall_chunk = -1;               // test hook (BSR_TEST_STALL_CHUNK at create): never load this X chunk
 };
 
 inline size_t dtype_size(bsr_dtype_t dt) { return dt == BSR_F32 ? 4 : 2; }
@@ -106,8 +113,13 @@ struct LaunchArgs {
     int *status;
     int64_t N;
     cudaStream_t stream;
+    uint64_t wait_ns;      // bound on every device-side wait
+    int stall_chunk;       // test hook, -1 in normal use
 };
 cudaError_t launch_generic(const LaunchArgs &a);
+cudaError_t launch_xstage(const LaunchArgs &a, int G);
+cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, float *wpk,
+                             cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);
 int launches_per_call(const Schedule &sc);
 

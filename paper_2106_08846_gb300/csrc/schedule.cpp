@@ -10,7 +10,9 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <numeric>
+#include <string>
 
 #include "schedule.h"
 
@@ -72,20 +74,76 @@ int64_t split_limit(const Schedule &sc) {
     return sc.max_row > limit ? limit : 0;
 }
 
+// For each task size G, the largest block-value and index footprint over
+// the tasks formed by G consecutive items of the (LPT-ordered) item list.
+void plan_xstage(Schedule &sc) {
+    const size_t per_block = (size_t)sc.R * sc.C * 4;
+    for (int gi = 0; gi < 4; gi++) {
+        const int G = 1 << gi;
+        size_t wmax = 0, imax = 0;
+        for (size_t t = 0; t < sc.items.size(); t += G) {
+            size_t blocks = 0;
+            for (size_t k = t; k < std::min(sc.items.size(), t + G); k++)
+                blocks += (size_t)(sc.items[k].p1 - sc.items[k].p0);
+            wmax = std::max(wmax, blocks * per_block);
+            imax = std::max(imax, blocks * 4);
+        }
+        sc.xs.task_wbytes[gi] = wmax;
+        sc.xs.task_ibytes[gi] = imax;
+    }
+    // per item, the first (item-local) block of each K chunk of kXsChunk columns
+    const int64_t nch = (sc.K + kXsChunk - 1) / kXsChunk;
+    sc.xs_cb.assign(sc.items.size() * (size_t)(nch + 1), 0);
+    for (size_t i = 0; i < sc.items.size(); i++) {
+        const Item &it = sc.items[i];
+        int32_t b = 0;
+        const int32_t len = it.p1 - it.p0;
+        for (int64_t c = 0; c <= nch; c++) {
+            const int64_t first_col = c * (kXsChunk / sc.C);
+            while (b < len && sc.indices[it.p0 + b] < first_col) b++;
+            sc.xs_cb[i * (size_t)(nch + 1) + c] = b;
+        }
+    }
+}
+
+const char *env_str(const char *name) {
+    const char *v = getenv(name);
+    return v && *v ? v : nullptr;
+}
+
 }  // namespace
 
 bsr_status_t build_schedule(Schedule &sc) {
     row_stats(sc);
-    sc.variant = V_GENERIC;
     sc.threads = 256;
-    sc.tn = std::max(1, 256 / std::min(sc.R, 256));
     sc.groups = 1;
     sc.smem = 0;
-    make_items(sc, split_limit(sc));
+    if (cudaDeviceGetAttribute(&sc.sm_count, cudaDevAttrMultiProcessorCount, sc.device) != cudaSuccess) {
+        cudaGetLastError();
+        sc.sm_count = 148;
+    }
+    const char *force = env_str("BSR_FORCE_VARIANT");
+    const bool want_generic = force && std::string(force) == "generic";
+    if (!want_generic && xstage_supports(sc.R, sc.C, sc.dt, sc.K)) {
+        sc.variant = V_XSTAGE;
+        sc.tn = kXsTokens;
+        sc.threads = (kXsConsumerWarps + 1) * 32;
+        const size_t budget = xstage_task_budget(sc.dt, sc.R, sc.K);
+        const int64_t lmax = std::max<int64_t>(1, (int64_t)(budget / ((size_t)sc.R * sc.C * 4 + 4)));
+        int64_t limit = split_limit(sc);
+        limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
+        make_items(sc, limit);
+        plan_xstage(sc);
+    } else {
+        sc.variant = V_GENERIC;
+        sc.tn = std::max(1, 256 / std::min(sc.R, 256));
+        make_items(sc, split_limit(sc));
+    }
     sc.group_begin = {0, (int32_t)sc.items.size()};
     if (upload(&sc.d_items, sc.items) != cudaSuccess || upload(&sc.d_splits, sc.splits) != cudaSuccess ||
         upload(&sc.d_group_begin, sc.group_begin) != cudaSuccess ||
-        upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess) {
+        upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess ||
+        upload(&sc.d_xs_cb, sc.xs_cb) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
@@ -94,13 +152,60 @@ bsr_status_t build_schedule(Schedule &sc) {
 
 bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
+    const Schedule &sc = *h.sched;
+    if (sc.variant != V_XSTAGE || sc.nnzb == 0) return BSR_OK;
+    const size_t bytes = (size_t)sc.nnzb * sc.R * sc.C * 4;
+    if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        h.data_packed = nullptr;
+        return BSR_ERR_ALLOC;
+    }
+    if (pack_xstage_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, (float *)h.data_packed, 0) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess) {
+        cudaGetLastError();
+        return BSR_ERR_CUDA;
+    }
     return BSR_OK;
 }
 
 int launches_per_call(const Schedule &sc) { return 1 + (sc.splits.empty() ? 0 : 1); }
 
+// Task size for this call: the largest G whose grid still gives every SM
+// `per_sm` CTAs, among those whose block values fit the shared-memory budget.
+int choose_tasks(const Schedule &sc, int64_t N) {
+    static const int per_sm = [] {
+        const char *v = getenv("BSR_XS_CTAS_PER_SM");
+        return v ? std::max(1, atoi(v)) : 2;
+    }();
+    static const int forced = [] {
+        const char *v = getenv("BSR_XS_G");
+        return v ? atoi(v) : 0;
+    }();
+    auto fits = [&](int G) {
+        const int gi = g_index(G);
+        return xstage_smem_bytes(sc.dt, sc.R, sc.K, G, sc.xs.task_wbytes[gi], sc.xs.task_ibytes[gi]) <=
+               (size_t)kXsMaxSmem;
+    };
+    if ((forced == 1 || forced == 2 || forced == 4 || forced == 8) && fits(forced)) return forced;
+    const int64_t tiles = (N + kXsTokens - 1) / kXsTokens;
+    const int64_t items = (int64_t)sc.items.size();
+    int best = 0;
+    for (int gi = 3; gi >= 0; gi--) {
+        const int G = 1 << gi;
+        if (!fits(G)) continue;
+        if (!best) best = G;   // largest that fits, if none reaches the target
+        if (tiles * ((items + G - 1) / G) >= (int64_t)per_sm * sc.sm_count) return G;
+        best = G;
+    }
+    return best ? best : 1;
+}
+
 cudaError_t launch_spmm(const LaunchArgs &a) {
-    cudaError_t e = launch_generic(a);
+    cudaError_t e;
+    if (a.sc->variant == V_XSTAGE)
+        e = launch_xstage(a, choose_tasks(*a.sc, a.N));
+    else
+        e = launch_generic(a);
     if (e != cudaSuccess) return e;
     if (!a.sc->splits.empty()) e = launch_reduce(a);
     return e;

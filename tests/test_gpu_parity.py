@@ -268,3 +268,28 @@ def test_error_statuses():
     assert lib.bsr_create(P(indptr.cpu().data_ptr()), P(indices.data_ptr()), P(data.data_ptr()), 8, 1, 128,
                           128, 0, ctypes.byref(out)) == b.BSR_ERR_INVALID_ARG
     assert h.check_device_status() == b.BSR_OK
+
+
+def test_bounded_wait_times_out_and_reports(monkeypatch):
+    """An X chunk that is never loaded: every wait on it gives up after the
+    bound (2 ms here), the kernel records BSR_ERR_TIMEOUT and returns; the
+    context stays usable and a normal handle still computes correctly."""
+    bsr = _bsr()
+    from paper_2106_08846_gb300 import bsrlib as b
+    w = _weight(256, 512, 32, 1, "f32", 0.2, 21)
+    gpu = build_on_gpu(w.W, 32, 1)
+    monkeypatch.setenv("BSR_WAIT_LIMIT_NS", "2000000")
+    monkeypatch.setenv("BSR_TEST_STALL_CHUNK", "1")
+    h = bsr.bsr_create(*gpu, 32, 1, 256, 512)
+    monkeypatch.delenv("BSR_WAIT_LIMIT_NS")
+    monkeypatch.delenv("BSR_TEST_STALL_CHUNK")
+    if h.schedule()["variant"] != "xstage":
+        pytest.skip("no bounded wait on this path")
+    X = synth.activations(22, 128, 512, "f32")
+    h.spmm(to_dev(X), to_dev(w.bias))
+    assert h.check_device_status() == b.BSR_ERR_TIMEOUT
+    assert h.check_device_status() == b.BSR_OK          # cleared after reading
+    h2 = bsr.bsr_create(*gpu, 32, 1, 256, 512)
+    Y = to_host(h2.spmm(to_dev(X), to_dev(w.bias)))
+    assert h2.check_device_status() == b.BSR_OK
+    check_product(Y, oracle.bsr_from_dense(w.W, 32, 1), X, w.bias, 256)
