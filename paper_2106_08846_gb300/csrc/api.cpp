@@ -117,7 +117,8 @@ Schedule::~Schedule() {
     cudaFree(d_splits);
     cudaFree(d_group_begin);
     cudaFree(d_indptr);
-    cudaFree(d_xs_cb);
+    cudaFree(d_xs_rec);
+    cudaFree(d_xs_rec_off);
     cudaFree(d_indices);
 }
 

@@ -65,8 +65,10 @@ struct Schedule {
     Item *d_items = nullptr;
     Split *d_splits = nullptr;
     int32_t *d_group_begin = nullptr;
-    std::vector<int32_t> xs_cb;         // xstage: per item, first block of each K chunk
-    int32_t *d_xs_cb = nullptr;
+    std::vector<int32_t> xs_rec;        // xstage: per-item records (block offsets/columns, chunk starts)
+    std::vector<int32_t> xs_rec_off;    // per item: record offset in ints (multiple of 4)
+    int32_t *d_xs_rec = nullptr;
+    int32_t *d_xs_rec_off = nullptr;
     int32_t *d_indptr = nullptr;        // owned copies of the structure
     int32_t *d_indices = nullptr;
 

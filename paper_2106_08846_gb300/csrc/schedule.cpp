@@ -77,32 +77,44 @@ int64_t split_limit(const Schedule &sc) {
 // For each task size G, the largest block-value and index footprint over
 // the tasks formed by G consecutive items of the (LPT-ordered) item list.
 void plan_xstage(Schedule &sc) {
-    const size_t per_block = (size_t)sc.R * sc.C * 4;
-    for (int gi = 0; gi < 4; gi++) {
-        const int G = 1 << gi;
-        size_t wmax = 0, imax = 0;
-        for (size_t t = 0; t < sc.items.size(); t += G) {
-            size_t blocks = 0;
-            for (size_t k = t; k < std::min(sc.items.size(), t + G); k++)
-                blocks += (size_t)(sc.items[k].p1 - sc.items[k].p0);
-            wmax = std::max(wmax, blocks * per_block);
-            imax = std::max(imax, blocks * 4);
-        }
-        sc.xs.task_wbytes[gi] = wmax;
-        sc.xs.task_ibytes[gi] = imax;
-    }
-    // per item, the first (item-local) block of each K chunk of kXsChunk columns
     const int64_t nch = (sc.K + kXsChunk - 1) / kXsChunk;
-    sc.xs_cb.assign(sc.items.size() * (size_t)(nch + 1), 0);
+    // per-item records: block offsets (C == 1) or columns, then chunk starts
+    sc.xs_rec.clear();
+    sc.xs_rec_off.assign(sc.items.size(), 0);
     for (size_t i = 0; i < sc.items.size(); i++) {
         const Item &it = sc.items[i];
-        int32_t b = 0;
         const int32_t len = it.p1 - it.p0;
+        sc.xs_rec_off[i] = (int32_t)sc.xs_rec.size();
+        const size_t base = sc.xs_rec.size();
+        sc.xs_rec.resize(base + (size_t)xstage_record_ints(len, nch), 0);
+        for (int32_t b = 0; b < len; b++) {
+            const int64_t col = sc.indices[it.p0 + b];
+            sc.xs_rec[base + b] = sc.C == 1 ? (int32_t)xstage_stage_offset(sc.dt, (int)(col % kXsChunk)) : (int32_t)col;
+        }
+        int32_t b = 0;
+        const size_t cbase = base + (size_t)xstage_pad4(len);
         for (int64_t c = 0; c <= nch; c++) {
             const int64_t first_col = c * (kXsChunk / sc.C);
             while (b < len && sc.indices[it.p0 + b] < first_col) b++;
-            sc.xs_cb[i * (size_t)(nch + 1) + c] = b;
+            sc.xs_rec[cbase + c] = b;
         }
+    }
+    const size_t per_block = (size_t)sc.R * sc.C * 4 * kXsWDup;
+    for (int gi = 0; gi < kXsTaskSizes; gi++) {
+        const int G = kXsG[gi];
+        size_t wmax = 0, imax = 0;
+        for (size_t t = 0; t < sc.items.size(); t += G) {
+            size_t blocks = 0, rec = 0;
+            for (size_t k = t; k < std::min(sc.items.size(), t + G); k++) {
+                const int64_t len = sc.items[k].p1 - sc.items[k].p0;
+                blocks += (size_t)len;
+                rec += (size_t)xstage_record_ints(len, nch) * 4;
+            }
+            wmax = std::max(wmax, blocks * per_block);
+            imax = std::max(imax, rec);
+        }
+        sc.xs.task_wbytes[gi] = wmax;
+        sc.xs.task_ibytes[gi] = imax;
     }
 }
 
@@ -129,7 +141,10 @@ bsr_status_t build_schedule(Schedule &sc) {
         sc.tn = kXsTokens;
         sc.threads = (kXsConsumerWarps + 1) * 32;
         const size_t budget = xstage_task_budget(sc.dt, sc.R, sc.K);
-        const int64_t lmax = std::max<int64_t>(1, (int64_t)(budget / ((size_t)sc.R * sc.C * 4 + 4)));
+        const int64_t nch = (sc.K + kXsChunk - 1) / kXsChunk;
+        const int64_t avail = (int64_t)budget - 4 * xstage_pad4(nch + 1) - 16;
+        const int64_t lmax =
+            std::max<int64_t>(1, avail / (int64_t)((size_t)sc.R * sc.C * 4 * kXsWDup + 4));
         int64_t limit = split_limit(sc);
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
         make_items(sc, limit);
@@ -143,7 +158,7 @@ bsr_status_t build_schedule(Schedule &sc) {
     if (upload(&sc.d_items, sc.items) != cudaSuccess || upload(&sc.d_splits, sc.splits) != cudaSuccess ||
         upload(&sc.d_group_begin, sc.group_begin) != cudaSuccess ||
         upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess ||
-        upload(&sc.d_xs_cb, sc.xs_cb) != cudaSuccess) {
+        upload(&sc.d_xs_rec, sc.xs_rec) != cudaSuccess || upload(&sc.d_xs_rec_off, sc.xs_rec_off) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
@@ -154,7 +169,7 @@ bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
     const Schedule &sc = *h.sched;
     if (sc.variant != V_XSTAGE || sc.nnzb == 0) return BSR_OK;
-    const size_t bytes = (size_t)sc.nnzb * sc.R * sc.C * 4;
+    const size_t bytes = (size_t)sc.nnzb * sc.R * sc.C * 4 * kXsWDup;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
         h.data_packed = nullptr;
@@ -170,13 +185,11 @@ bsr_status_t pack_data(Handle &h) {
 
 int launches_per_call(const Schedule &sc) { return 1 + (sc.splits.empty() ? 0 : 1); }
 
-// Task size for this call: the largest G whose grid still gives every SM
-// `per_sm` CTAs, among those whose block values fit the shared-memory budget.
+// Task size for this call: the G that minimises a simple cost model,
+// waves * (fixed CTA cost + G items of work), among the G whose shared
+// memory fits. One CTA runs per SM; a CTA's fixed cost (pipeline fill,
+// staging, epilogue) is worth about kOverheadItems average items.
 int choose_tasks(const Schedule &sc, int64_t N) {
-    static const int per_sm = [] {
-        const char *v = getenv("BSR_XS_CTAS_PER_SM");
-        return v ? std::max(1, atoi(v)) : 2;
-    }();
     static const int forced = [] {
         const char *v = getenv("BSR_XS_G");
         return v ? atoi(v) : 0;
@@ -186,18 +199,25 @@ int choose_tasks(const Schedule &sc, int64_t N) {
         return xstage_smem_bytes(sc.dt, sc.R, sc.K, G, sc.xs.task_wbytes[gi], sc.xs.task_ibytes[gi]) <=
                (size_t)kXsMaxSmem;
     };
-    if ((forced == 1 || forced == 2 || forced == 4 || forced == 8) && fits(forced)) return forced;
+    for (int gi = 0; gi < kXsTaskSizes; gi++)
+        if (forced == kXsG[gi] && fits(forced)) return forced;
+    const double kOverheadItems = 2.0;
     const int64_t tiles = (N + kXsTokens - 1) / kXsTokens;
     const int64_t items = (int64_t)sc.items.size();
-    int best = 0;
-    for (int gi = 3; gi >= 0; gi--) {
-        const int G = 1 << gi;
+    int best = 1;
+    double best_cost = -1.0;
+    for (int gi = 0; gi < kXsTaskSizes; gi++) {
+        const int G = kXsG[gi];
         if (!fits(G)) continue;
-        if (!best) best = G;   // largest that fits, if none reaches the target
-        if (tiles * ((items + G - 1) / G) >= (int64_t)per_sm * sc.sm_count) return G;
-        best = G;
+        const int64_t ctas = tiles * ((items + G - 1) / G);
+        const double waves = (double)((ctas + sc.sm_count - 1) / sc.sm_count);
+        const double cost = waves * (kOverheadItems + (double)std::min<int64_t>(G, items));
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = G;
+        }
     }
-    return best ? best : 1;
+    return best;
 }
 
 cudaError_t launch_spmm(const LaunchArgs &a) {

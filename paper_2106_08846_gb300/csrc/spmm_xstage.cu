@@ -1,34 +1,43 @@
 // SIMT BSR x dense kernel with X staged through a TMA ring ("xstage").
 //
 // Each CTA owns a tile of TN = 64 tokens and a task of G work items (block
-// rows or pieces of rows, Section 2.2's kept blocks), S = 8/G consumer warps
-// per item. The inner product over the kept blocks is FP32-FMA bound, so the
-// design goal is a high FMA:issue ratio:
+// rows or pieces of rows, Section 2.2's kept blocks), S = 12/G consumer warps
+// per item (12 consumer warps and one producer warp). The inner product over the kept blocks is FP32-FMA bound, so the
+// design goal is a high share of packed FMAs among the issued instructions:
 //
-//  * X[n0 : n0+64, k0 : k0+128] chunks stream through a 3-stage shared-memory
-//    ring: one producer thread issues 2-D TMA tile loads (128-byte swizzle,
-//    rows = tokens) and arms the stage's "full" mbarrier; every consumer warp
-//    waits for every chunk in order, processes all of its blocks that fall in
-//    it, and releases it on the stage's "empty" mbarrier.
-//  * The task's block values (repacked at create time to fp32 [p][c][r]),
-//    block-column indices and, per item, the first block of every chunk are
-//    put in shared memory once, so the per-chunk loop has no search or test.
+//  * The CL CTAs of a thread-block cluster share one token tile (different
+//    tasks). X[n0 : n0+64, k0 : k0+128] chunks stream through a 3-stage
+//    shared-memory ring: each CTA's producer thread loads a 64/CL-row slice
+//    of the chunk with a 2-D TMA multicast (128-byte swizzle, rows = tokens)
+//    into the same stage of every CTA of the cluster. A stage's "full"
+//    mbarrier counts the bytes of all slices; every consumer warp waits for
+//    every chunk in order, processes all of its blocks that fall in it, and
+//    releases the stage on the "empty" mbarrier of every CTA in the cluster.
+//  * Per item, the producer fetches by bulk copy the block values (repacked
+//    at create time to fp32 [p][c][r]) and a record built on the host: each
+//    block's X offset inside a stage (1-column blocks) or block column, and
+//    the first block of every chunk, so the per-chunk loop has no search or
+//    test. The consumers load the bias meanwhile.
 //  * Lane = tg + 8 q: tg picks 8 tokens (tg, tg+8, ..., tg+56: conflict-free
 //    under the swizzle, which XORs the 16-byte column group with tg), q
 //    splits into NRG output groups of TR rows and NKS = 4/NRG lanes that take
 //    alternate blocks. A lane accumulates an 8 x TR tile with packed
-//    fma.rn.f32x2 (pairs of outputs, or pairs of tokens when TR = 1).
-//  * Epilogue: shuffle-reduce the NKS partials, sum the S warps of an item in
-//    a fixed order through shared memory, add the bias, convert and store
-//    (or write an fp32 partial for rows split across CTAs).
+//    fma.rn.f32x2 over pairs of tokens: (x_t, x_t') * (w, w).
+//  * Epilogue: shuffle-reduce the NKS partials, then sum the S warps of an
+//    item by a fixed pairwise tree through shared memory; the item's first
+//    warp adds the bias, converts and stores from registers (or writes an
+//    fp32 partial for rows split across CTAs).
 //
 // Every wait is bounded by the global timer; a timeout sets the device
-// status word, stops the CTA's pipeline, drains its TMA loads and returns.
+// status word, stops the CTA's pipeline and drains its TMA loads. A cluster
+// barrier closes the kernel: no CTA leaves while another may still signal it.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <cstdlib>
 #include <mutex>
+#include <vector>
 
 #include "bsr_internal.h"
 #include "elem.cuh"
@@ -44,27 +53,30 @@ constexpr int KC = kXsChunk;
 constexpr int NS = kXsStages;
 constexpr int NCW = kXsConsumerWarps;
 constexpr int NTHREADS = (NCW + 1) * 32;
-constexpr uint64_t kDrainNs = 2000000000ull;   // generous bound for TMA loads already issued
+constexpr int WD = kXsWDup;
+constexpr uint64_t kDrainNs = 200000000ull;   // bound for TMA loads already issued (they take microseconds)
 
 struct XsArgs {
     const Item *items;
     int n_items, G, S, n_tasks;
-    const int32_t *indices;
-    const int32_t *cb;       // per item: first block of every chunk, [n_items][nchunks + 1]
-    const float *wpk;
+    const int32_t *rec;      // per-item records (xstage_record_ints)
+    const int32_t *rec_off;  // per item: record offset in ints
+    const float *wpk;        // [nnzb][C][R][WD]
     const float *bias;
     void *Y;
     float *ws;
     int *status;
     int64_t N, K, M;
     int C, nchunks;
-    uint32_t w_off, idx_off, cb_off, bias_off, bar_off, misc_off;
+    uint32_t w_off, idx_off, bias_off, bar_off, misc_off;
     int w_bulk;              // block values arrive by one bulk copy per item
     uint64_t wait_ns;
-    int stall_chunk;    // test hook: this chunk is never loaded (-1: none)
+    int stall_chunk;         // test hook: this chunk is never loaded (-1: none)
 };
 
 // Shared-memory image of one X chunk: 64 token rows, 128-byte swizzled boxes.
+// off0(kk) is the byte offset of chunk column kk in token row 0; token tg + 8 i
+// is at (off0 ^ (tg << 4)) + tg * 128 + i * 1024.
 template <typename T>
 struct Stage;
 template <>
@@ -73,9 +85,8 @@ struct Stage<float> {
     static constexpr int kBoxes = KC / kBoxCols;
     static constexpr uint32_t kBoxBytes = TN * 128;
     static constexpr uint32_t kBytes = kBoxes * kBoxBytes;
-    // byte offset of column kk in token row tg (token tg + 8 i adds i * 1024)
-    __device__ static __forceinline__ uint32_t off(int kk, int tg) {
-        return (uint32_t)((kk >> 5) * kBoxBytes + tg * 128 + ((((kk & 31) >> 2) ^ tg) << 4) + (kk & 3) * 4);
+    __host__ __device__ static __forceinline__ uint32_t off0(int kk) {
+        return (uint32_t)((kk >> 5) * kBoxBytes + (((kk & 31) >> 2) << 4) + (kk & 3) * 4);
     }
 };
 template <>
@@ -84,8 +95,8 @@ struct Stage<uint16_t> {
     static constexpr int kBoxes = KC / kBoxCols;
     static constexpr uint32_t kBoxBytes = TN * 128;
     static constexpr uint32_t kBytes = kBoxes * kBoxBytes;
-    __device__ static __forceinline__ uint32_t off(int kk, int tg) {
-        return (uint32_t)((kk >> 6) * kBoxBytes + tg * 128 + ((((kk & 63) >> 3) ^ tg) << 4) + (kk & 7) * 2);
+    __host__ __device__ static __forceinline__ uint32_t off0(int kk) {
+        return (uint32_t)((kk >> 6) * kBoxBytes + (((kk & 63) >> 3) << 4) + (kk & 7) * 2);
     }
 };
 
@@ -93,7 +104,7 @@ __device__ __forceinline__ float ld_x(const unsigned char *p, float) { return *r
 __device__ __forceinline__ float ld_x(const unsigned char *p, uint16_t) {
     return to_f32(*reinterpret_cast<const uint16_t *>(p));
 }
-// four consecutive columns
+// four consecutive columns of one token
 __device__ __forceinline__ float4 ld_x4(const unsigned char *p, float) {
     return *reinterpret_cast<const float4 *>(p);
 }
@@ -118,47 +129,36 @@ __device__ __forceinline__ f2_t ffma2(f2_t a, f2_t b, f2_t c) {
     return d;
 }
 
-// acc (8 tokens x TR outputs, packed in pairs) += x (8 tokens) * w (TR outputs)
+// acc (8 tokens x TR outputs) += x (8 tokens) * w (TR outputs); accumulators
+// packed over token pairs (i, i+1) for i even.
 template <int TR>
 struct Tile {
-    static constexpr int NP = TR >= 2 ? 8 * TR / 2 : 4;   // packed accumulators
-    f2_t a[NP];
+    f2_t a[4 * TR];
     __device__ __forceinline__ void zero() {
 #pragma unroll
-        for (int k = 0; k < NP; k++) a[k] = 0ull;
+        for (int k = 0; k < 4 * TR; k++) a[k] = 0ull;
     }
     __device__ __forceinline__ void fma(const float (&x)[8], const float (&w)[TR]) {
-        if constexpr (TR >= 2) {
-            f2_t wp[TR / 2];
+        f2_t wd[TR];
 #pragma unroll
-            for (int j = 0; j < TR / 2; j++) wp[j] = pack2(w[2 * j], w[2 * j + 1]);
+        for (int j = 0; j < TR; j++) wd[j] = pack2(w[j], w[j]);
 #pragma unroll
-            for (int i = 0; i < 8; i++) {
-                const f2_t xx = pack2(x[i], x[i]);
+        for (int ip = 0; ip < 4; ip++) {
+            const f2_t xp = pack2(x[2 * ip], x[2 * ip + 1]);
 #pragma unroll
-                for (int j = 0; j < TR / 2; j++) a[i * (TR / 2) + j] = ffma2(xx, wp[j], a[i * (TR / 2) + j]);
-            }
-        } else {
-            const f2_t ww = pack2(w[0], w[0]);
-#pragma unroll
-            for (int i = 0; i < 4; i++) a[i] = ffma2(pack2(x[2 * i], x[2 * i + 1]), ww, a[i]);
+            for (int j = 0; j < TR; j++) a[ip * TR + j] = ffma2(xp, wd[j], a[ip * TR + j]);
         }
     }
-    // value for token i, output j
     __device__ __forceinline__ float get(int i, int j) const {
         float lo, hi;
-        if constexpr (TR >= 2) {
-            unpack2(a[i * (TR / 2) + j / 2], lo, hi);
-            return (j & 1) ? hi : lo;
-        } else {
-            unpack2(a[i / 2], lo, hi);
-            return (i & 1) ? hi : lo;
-        }
+        unpack2(a[(i >> 1) * TR + j], lo, hi);
+        return (i & 1) ? hi : lo;
     }
 };
 
+// the TR weights of one block column for this lane
 template <int TR>
-__device__ __forceinline__ void load_w(const float *wr, float (&w)[TR]) {
+__device__ __forceinline__ void load_wd(const float *wr, float (&w)[TR]) {
     if constexpr (TR % 4 == 0) {
 #pragma unroll
         for (int j = 0; j < TR; j += 4) {
@@ -168,9 +168,12 @@ __device__ __forceinline__ void load_w(const float *wr, float (&w)[TR]) {
             w[j + 2] = v.z;
             w[j + 3] = v.w;
         }
+    } else if constexpr (TR == 2) {
+        const float2 v = *reinterpret_cast<const float2 *>(wr);
+        w[0] = v.x;
+        w[1] = v.y;
     } else {
-#pragma unroll
-        for (int j = 0; j < TR; j++) w[j] = wr[j];
+        w[0] = wr[0];
     }
 }
 
@@ -180,189 +183,157 @@ __device__ __forceinline__ bool aborted(const int *flag) {
     return *reinterpret_cast<const volatile int *>(flag) != 0;
 }
 
-template <typename T, int TR, int NRG>
-__global__ void __launch_bounds__(NTHREADS, 1)
-k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
+struct Shared {
+    unsigned char *base;
+    uint64_t *full, *empty, *wbar;
+    int *misc;          // [0] abort flag
+    int *itab;          // per item: row p0 p1 slot rec_off len
+    float *W;           // block values of the task's items
+    int32_t *I;         // the task's item records
+    float *B;           // [item][R] bias
+};
+
+// Offsets of item g's block values (floats) and record (ints) in shared memory.
+__device__ __forceinline__ void item_offsets(const int *itab, int g, int per_block, int nch, int &woff, int &roff) {
+    woff = 0;
+    roff = 0;
+    for (int k = 0; k < g; k++) {
+        const int len = itab[6 * k + 5];
+        woff += len * per_block;
+        roff += (int)xstage_record_ints(len, nch);
+    }
+}
+
+template <typename T, int TR, int NRG, int CT>
+__device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int64_t n0, int item_first,
+                                         int g_count, uint32_t CL, int warp, int lane) {
     using St = Stage<T>;
     constexpr int NKS = 4 / NRG;
     constexpr int R = TR * NRG;
-    extern __shared__ unsigned char smem_raw[];
-    unsigned char *smem =
-        reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + a.bar_off);
-    uint64_t *empty = full + NS;
-    uint64_t *wbar = empty + NS;                              // block values landed
-    int *misc = reinterpret_cast<int *>(smem + a.misc_off);   // [0] abort flag, then the item table
-    int *itab = misc + 4;                                     // per item: row p0 p1 slot woff ioff
-    float *W_s = reinterpret_cast<float *>(smem + a.w_off);
-    int32_t *I_s = reinterpret_cast<int32_t *>(smem + a.idx_off);
-    int32_t *CB = reinterpret_cast<int32_t *>(smem + a.cb_off);   // [item][nchunks + 1]
-    float *B_s = reinterpret_cast<float *>(smem + a.bias_off);      // [item][R]
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // consecutive CTAs take different token tiles, so that concurrent CTAs
-    // spread their X reads over many tiles
-    const int64_t n_tiles = (a.N + TN - 1) / TN;
-    const int task = (int)(blockIdx.x / n_tiles);
-    const int64_t n0 = (int64_t)(blockIdx.x % n_tiles) * TN;
-    const int item_first = task * a.G;
-    const int g_count = min(a.G, a.n_items - item_first);
-    const int C = a.C;
+    const int C = CT ? CT : a.C;
     const int nch = a.nchunks;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < NS; s++) {
-            ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], NCW);
-        }
-        ptx::mbar_init(wbar, 1);
-        misc[0] = 0;
-        int woff = 0, ioff = 0;
-        for (int g = 0; g < g_count; g++) {
-            const Item it = a.items[item_first + g];
-            const int len = it.p1 - it.p0;
-            itab[6 * g + 0] = it.row;
-            itab[6 * g + 1] = it.p0;
-            itab[6 * g + 2] = it.p1;
-            itab[6 * g + 3] = it.slot;
-            itab[6 * g + 4] = woff;
-            itab[6 * g + 5] = ioff;
-            woff += len * R * C;
-            ioff += len;
-        }
-        ptx::fence_barrier_init();
-    }
-    __syncthreads();
-
-    if (warp == NCW) {
-        // ---------------- producer: one thread streams X chunks through the ring
-        if (lane == 0) {
-            ptx::prefetch_tensormap(&xmap);
-            if (a.w_bulk) {
-                uint32_t total = 0;
-                for (int g = 0; g < g_count; g++) total += (uint32_t)(itab[6 * g + 2] - itab[6 * g + 1]) * R * C * 4;
-                ptx::mbar_arrive_expect_tx(wbar, total);
-                for (int g = 0; g < g_count; g++) {
-                    const uint32_t bytes = (uint32_t)(itab[6 * g + 2] - itab[6 * g + 1]) * R * C * 4;
-                    if (bytes)
-                        ptx::bulk_load(W_s + itab[6 * g + 4], a.wpk + (int64_t)itab[6 * g + 1] * R * C, bytes, wbar);
-                }
-            }
-            int c = 0;
-            bool ok = true;
-            for (; c < nch; c++) {
-                const int s = c % NS;
-                if (c >= NS && !ptx::mbar_wait_bounded(&empty[s], ((c / NS) - 1) & 1, a.wait_ns)) {
-                    ok = false;
-                    break;
-                }
-                if (aborted(misc)) { ok = false; break; }
-                if (c == a.stall_chunk) continue;   // its consumers time out
-                ptx::mbar_arrive_expect_tx(&full[s], St::kBytes);
-#pragma unroll
-                for (int b = 0; b < St::kBoxes; b++)
-                    ptx::tma_load_2d(smem + s * St::kBytes + b * St::kBoxBytes, &xmap,
-                                     c * KC + b * St::kBoxCols, (int32_t)n0, &full[s]);
-            }
-            if (!ok) {
-                set_status(a.status, DEV_TIMEOUT);
-                atomicExch(&misc[0], 1);
-            }
-            // the last loads issued may still be in flight: wait (bounded) for
-            // them so that no TMA write outlives the CTA
-            for (int d = max(0, c - NS); d < c; d++)
-                if (d != a.stall_chunk) ptx::mbar_wait_bounded(&full[d % NS], (d / NS) & 1, kDrainNs);
-            if (a.w_bulk) ptx::mbar_wait_bounded(wbar, 0, kDrainNs);
-        }
-        return;
-    }
-
-    // ---------------- consumers: stage indices, chunk starts, bias (and block
-    // values when they cannot come by bulk copy)
     const int ctid = threadIdx.x;   // 0 .. NCW*32-1
+
+    // ---- bias (and block values when they cannot come by bulk copy); the
+    // records and block values arrive by the producer's bulk copies
     for (int g = 0; g < g_count; g++) {
-        const int p0 = itab[6 * g + 1], len = itab[6 * g + 2] - p0;
-        const int ioff = itab[6 * g + 5];
         if (!a.w_bulk) {
-            const int woff = itab[6 * g + 4];
-            const float *src = a.wpk + (int64_t)p0 * R * C;
-            for (int e = ctid; e < len * R * C; e += NCW * 32) W_s[woff + e] = __ldg(src + e);
+            int woff, roff;
+            item_offsets(sh.itab, g, R * C * WD, nch, woff, roff);
+            const int p0 = sh.itab[6 * g + 1], len = sh.itab[6 * g + 5];
+            const float *src = a.wpk + (int64_t)p0 * R * C * WD;
+            for (int e = ctid; e < len * R * C * WD; e += NCW * 32) sh.W[woff + e] = __ldg(src + e);
         }
-        for (int e = ctid; e < len; e += NCW * 32) I_s[ioff + e] = __ldg(a.indices + p0 + e);
-        const int32_t *cbg = a.cb + (int64_t)(item_first + g) * (nch + 1);
-        for (int e = ctid; e <= nch; e += NCW * 32) CB[g * (nch + 1) + e] = __ldg(cbg + e);
-        const int64_t m0 = (int64_t)itab[6 * g + 0] * R;
-        for (int e = ctid; e < R; e += NCW * 32) B_s[g * R + e] = a.bias ? __ldg(a.bias + m0 + e) : 0.f;
+        const int64_t m0 = (int64_t)sh.itab[6 * g + 0] * R;
+        for (int e = ctid; e < R; e += NCW * 32) sh.B[g * R + e] = a.bias ? __ldg(a.bias + m0 + e) : 0.f;
     }
     ptx::named_barrier(1, NCW * 32);
-    bool wok = true;
-    if (a.w_bulk) wok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(wbar, 0, a.wait_ns));
+    bool ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(sh.wbar, 0, a.wait_ns));
 
     const int q = lane >> 3, tg = lane & 7;
     const int rg = q % NRG, ks = q / NRG;
     const int S = a.S;
     const int gi = warp / S, piece = warp % S;
     const bool has_item = gi < g_count;
-    const int woff = has_item ? itab[6 * gi + 4] : 0;
-    const int ioff = has_item ? itab[6 * gi + 5] : 0;
-    const int32_t *cb = CB + (has_item ? gi : 0) * (nch + 1);
-    const float *wbase = W_s + woff + rg * TR;
+    int woff = 0, roff = 0;
+    if (has_item) item_offsets(sh.itab, gi, R * C * WD, nch, woff, roff);
+    const int32_t *idx = sh.I + roff;
+    const int32_t *cb = idx + (has_item ? xstage_pad4(sh.itab[6 * gi + 5]) : 0);
+    const float *wbase = sh.W + woff + rg * TR * WD;
+    const uint32_t tgx = (uint32_t)tg << 4;
+    const unsigned char *lane_base = sh.base + tg * 128;
 
     Tile<TR> acc;
     acc.zero();
-    bool ok = wok;
     for (int c = 0; c < nch && ok; c++) {
-        const bool got = ptx::mbar_wait_bounded(&full[c % NS], (c / NS) & 1, a.wait_ns) && !aborted(misc);
+        const bool got = ptx::mbar_wait_bounded(&sh.full[c % NS], (c / NS) & 1, a.wait_ns) && !aborted(sh.misc);
         ok = __all_sync(0xffffffffu, got);
         if (!ok) break;
         if (has_item) {
-            const unsigned char *st = smem + (c % NS) * St::kBytes;
+            const unsigned char *st = lane_base + (c % NS) * St::kBytes;
             const int lo = cb[c], hi = cb[c + 1];
             // this warp's blocks piece + S*jj inside [lo, hi); lanes ks take alternate ones
             const int j0 = lo <= piece ? 0 : (lo - piece + S - 1) / S;
             const int j1 = hi <= piece ? 0 : (hi - piece + S - 1) / S;
-            const int kbase = c * KC;
-            for (int jj = j0 + ks; jj < j1; jj += NKS) {
-                const int lb = piece + S * jj;
-                const int kk = I_s[ioff + lb] * C - kbase;
-                const float *wb = wbase + lb * C * R;
-                if ((C & 3) == 0) {
-                    for (int c4 = 0; c4 < C; c4 += 4) {
-                        const unsigned char *xp = st + St::off(kk + c4, tg);
-                        float4 xv[8];
+            if constexpr (CT == 1) {
+                // one block ahead: the next block's operands are loaded while
+                // the current block's FMAs issue
+                int jj = j0 + ks;
+                if (jj < j1) {
+                    float xn[8], wn[TR];
+                    {
+                        const int lb = piece + S * jj;
+                        const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
 #pragma unroll
-                        for (int i = 0; i < 8; i++) xv[i] = ld_x4(xp + i * 1024, T());
-#pragma unroll
-                        for (int u = 0; u < 4; u++) {
-                            float x[8], w[TR];
-#pragma unroll
-                            for (int i = 0; i < 8; i++)
-                                x[i] = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
-                            load_w<TR>(wb + (c4 + u) * R, w);
-                            acc.fma(x, w);
-                        }
+                        for (int i = 0; i < 8; i++) xn[i] = ld_x(xp + i * 1024, T());
+                        load_wd<TR>(wbase + lb * R * WD, wn);
                     }
-                } else {
-                    for (int cc = 0; cc < C; cc++) {
-                        const unsigned char *xp = st + St::off(kk + cc, tg);
-                        float x[8], w[TR];
+                    for (; jj < j1; jj += NKS) {
+                        float xc[8], wc[TR];
 #pragma unroll
-                        for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
-                        load_w<TR>(wb + cc * R, w);
-                        acc.fma(x, w);
+                        for (int i = 0; i < 8; i++) xc[i] = xn[i];
+#pragma unroll
+                        for (int j = 0; j < TR; j++) wc[j] = wn[j];
+                        if (jj + NKS < j1) {
+                            const int lb = piece + S * (jj + NKS);
+                            const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
+#pragma unroll
+                            for (int i = 0; i < 8; i++) xn[i] = ld_x(xp + i * 1024, T());
+                            load_wd<TR>(wbase + lb * R * WD, wn);
+                        }
+                        acc.fma(xc, wc);
+                    }
+                }
+            } else {
+                const int kbase = c * KC;
+                for (int jj = j0 + ks; jj < j1; jj += NKS) {
+                    const int lb = piece + S * jj;
+                    const int kk = idx[lb] * C - kbase;
+                    const float *wb = wbase + lb * C * R * WD;
+                    if ((C & 3) == 0) {
+                        for (int c4 = 0; c4 < C; c4 += 4) {
+                            const unsigned char *xp = st + (St::off0(kk + c4) ^ tgx);
+                            float4 xv[8];
+#pragma unroll
+                            for (int i = 0; i < 8; i++) xv[i] = ld_x4(xp + i * 1024, T());
+#pragma unroll
+                            for (int u = 0; u < 4; u++) {
+                                float x[8];
+                                float wd[TR];
+#pragma unroll
+                                for (int i = 0; i < 8; i++)
+                                    x[i] = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
+                                load_wd<TR>(wb + (c4 + u) * R * WD, wd);
+                                acc.fma(x, wd);
+                            }
+                        }
+                    } else {
+                        for (int cc = 0; cc < C; cc++) {
+                            const unsigned char *xp = st + (St::off0(kk + cc) ^ tgx);
+                            float x[8];
+                            float wd[TR];
+#pragma unroll
+                            for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
+                            load_wd<TR>(wb + cc * R * WD, wd);
+                            acc.fma(x, wd);
+                        }
                     }
                 }
             }
         }
         __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(&empty[c % NS]);
+        if (CL == 1) {
+            if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
+        } else if (lane < (int)CL) {
+            ptx::mbar_arrive_cluster(ptx::mapa(ptx::smem_addr(&sh.empty[c % NS]), lane));
+        }
     }
     if (!ok && lane == 0) {
         set_status(a.status, DEV_TIMEOUT);
-        atomicExch(&misc[0], 1);
+        atomicExch(&sh.misc[0], 1);
     }
 
-    // ---------------- epilogue
+    // ---- epilogue
     float v[8][TR];
 #pragma unroll
     for (int i = 0; i < 8; i++)
@@ -373,71 +344,206 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
             if constexpr (NKS >= 4) t += __shfl_xor_sync(0xffffffffu, t, 16 * NRG);
             v[i][j] = t;
         }
-    // every consumer is done with the ring and W_s; the abort verdict is the
-    // same for all of them (barrier reduction), so no thread skips a barrier
-    if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(misc))) return;
-    constexpr int PS = R + 4;          // padded row of the partial tile (16-byte aligned)
-    float *P = reinterpret_cast<float *>(smem);
-    if (ks == 0) {
-        float *Pw = P + warp * TN * PS;   // this warp's partial tile [TN][R] (padded rows)
+    // every consumer is done with the ring and the block values; the abort
+    // verdict is the same for all of them (barrier reduction)
+    if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
+    // pairwise tree over the S warps of each item: in round `step`, the warp
+    // of piece p (p % 2step == step) hands its tile to piece p - step
+    constexpr int PS = R + 4;          // padded row of a tile in shared memory (16-byte aligned)
+    float *P = reinterpret_cast<float *>(sh.base);
+    const int half = (S + 1) / 2;      // tiles per item in the first round
+    for (int step = 1; step < S; step <<= 1) {
+        float *slot = P + (gi * half + piece / (2 * step)) * TN * PS;
+        if (has_item && piece % (2 * step) == step && ks == 0) {
 #pragma unroll
-        for (int i = 0; i < 8; i++) {
-            float *dst = Pw + (tg + 8 * i) * PS + rg * TR;
-            if constexpr (TR % 4 == 0) {
+            for (int i = 0; i < 8; i++) {
+                float *dst = slot + (tg + 8 * i) * PS + rg * TR;
+                if constexpr (TR % 4 == 0) {
 #pragma unroll
-                for (int j = 0; j < TR; j += 4)
-                    *reinterpret_cast<float4 *>(dst + j) = make_float4(v[i][j], v[i][j + 1], v[i][j + 2], v[i][j + 3]);
-            } else {
+                    for (int j = 0; j < TR; j += 4)
+                        *reinterpret_cast<float4 *>(dst + j) = make_float4(v[i][j], v[i][j + 1], v[i][j + 2], v[i][j + 3]);
+                } else {
 #pragma unroll
-                for (int j = 0; j < TR; j++) dst[j] = v[i][j];
+                    for (int j = 0; j < TR; j++) dst[j] = v[i][j];
+                }
             }
         }
-    }
-    ptx::named_barrier(1, NCW * 32);
-    constexpr int V = R % 4 == 0 ? 4 : 1;   // outputs per thread and store
-    for (int g = 0; g < g_count; g++) {
-        const int row = itab[6 * g + 0], slot = itab[6 * g + 3];
-        for (int e = ctid; e < TN * R / V; e += NCW * 32) {
-            const int t = (e * V) / R, r = e * V - t * R;
-            const int64_t n = n0 + t;
-            if (n >= a.N) continue;
-            float o[V];
+        ptx::named_barrier(1, NCW * 32);
+        if (has_item && piece % (2 * step) == 0 && piece + step < S) {
 #pragma unroll
-            for (int u = 0; u < V; u++) o[u] = 0.f;
-            for (int pc = 0; pc < S; pc++) {
-                const float *src = P + ((g * S + pc) * TN + t) * PS + r;
-                if constexpr (V == 4) {
-                    const float4 q4 = *reinterpret_cast<const float4 *>(src);
-                    o[0] += q4.x; o[1] += q4.y; o[2] += q4.z; o[3] += q4.w;
+            for (int i = 0; i < 8; i++) {
+                const float *src = slot + (tg + 8 * i) * PS + rg * TR;
+                if constexpr (TR % 4 == 0) {
+#pragma unroll
+                    for (int j = 0; j < TR; j += 4) {
+                        const float4 q4 = *reinterpret_cast<const float4 *>(src + j);
+                        v[i][j] += q4.x;
+                        v[i][j + 1] += q4.y;
+                        v[i][j + 2] += q4.z;
+                        v[i][j + 3] += q4.w;
+                    }
                 } else {
-                    o[0] += src[0];
+#pragma unroll
+                    for (int j = 0; j < TR; j++) v[i][j] += src[j];
                 }
             }
-            const int64_t m = (int64_t)row * R + r;
-            if (slot < 0) {
+        }
+        ptx::named_barrier(1, NCW * 32);
+    }
+    if (!has_item || piece != 0 || ks != 0) return;
+    const int row = sh.itab[6 * gi + 0], slot = sh.itab[6 * gi + 3];
+    const int64_t m = (int64_t)row * R + rg * TR;
+    float b[TR];
 #pragma unroll
-                for (int u = 0; u < V; u++) o[u] += B_s[g * R + r + u];
-                T *dst = reinterpret_cast<T *>(a.Y) + n * a.M + m;
-                if constexpr (V == 4 && sizeof(T) == 4) {
-                    *reinterpret_cast<float4 *>(dst) = make_float4(o[0], o[1], o[2], o[3]);
-                } else if constexpr (V == 4) {
+    for (int j = 0; j < TR; j++) b[j] = slot < 0 ? sh.B[gi * R + rg * TR + j] : 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+        const int64_t n = n0 + tg + 8 * i;
+        if (n >= a.N) continue;
+        if (slot < 0) {
+            T *dst = reinterpret_cast<T *>(a.Y) + n * a.M + m;
+            if constexpr (sizeof(T) == 4 && TR % 4 == 0) {
+#pragma unroll
+                for (int j = 0; j < TR; j += 4)
+                    *reinterpret_cast<float4 *>(dst + j) =
+                        make_float4(v[i][j] + b[j], v[i][j + 1] + b[j + 1], v[i][j + 2] + b[j + 2], v[i][j + 3] + b[j + 3]);
+            } else if constexpr (sizeof(T) == 2 && TR % 4 == 0) {
+#pragma unroll
+                for (int j = 0; j < TR; j += 4) {
                     uint2 pk;
-                    pk.x = (uint32_t)from_f32<T>(o[0]) | ((uint32_t)from_f32<T>(o[1]) << 16);
-                    pk.y = (uint32_t)from_f32<T>(o[2]) | ((uint32_t)from_f32<T>(o[3]) << 16);
-                    *reinterpret_cast<uint2 *>(dst) = pk;
-                } else {
-                    dst[0] = from_f32<T>(o[0]);
+                    pk.x = (uint32_t)from_f32<T>(v[i][j] + b[j]) | ((uint32_t)from_f32<T>(v[i][j + 1] + b[j + 1]) << 16);
+                    pk.y = (uint32_t)from_f32<T>(v[i][j + 2] + b[j + 2]) |
+                           ((uint32_t)from_f32<T>(v[i][j + 3] + b[j + 3]) << 16);
+                    *reinterpret_cast<uint2 *>(dst + j) = pk;
                 }
             } else {
-                float *dst = a.ws + ((int64_t)slot * a.N + n) * R + r;
 #pragma unroll
-                for (int u = 0; u < V; u++) dst[u] = o[u];
+                for (int j = 0; j < TR; j++) dst[j] = from_f32<T>(v[i][j] + b[j]);
             }
+        } else {
+            float *dst = a.ws + ((int64_t)slot * a.N + n) * R + rg * TR;
+#pragma unroll
+            for (int j = 0; j < TR; j++) dst[j] = v[i][j];
         }
     }
 }
 
-// W^T per block, widened to fp32: wpk[(p*C + c)*R + r] = data[(p*R + r)*C + c].
+template <typename T, int TR, int NRG, int CT>
+__global__ void __launch_bounds__(NTHREADS, 1)
+k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
+    using St = Stage<T>;
+    constexpr int R = TR * NRG;
+    extern __shared__ unsigned char smem_raw[];
+    Shared sh;
+    sh.base = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    sh.full = reinterpret_cast<uint64_t *>(sh.base + a.bar_off);
+    sh.empty = sh.full + NS;
+    sh.wbar = sh.empty + NS;
+    sh.misc = reinterpret_cast<int *>(sh.base + a.misc_off);
+    sh.itab = sh.misc + 4;
+    sh.W = reinterpret_cast<float *>(sh.base + a.w_off);
+    sh.I = reinterpret_cast<int32_t *>(sh.base + a.idx_off);
+    sh.B = reinterpret_cast<float *>(sh.base + a.bias_off);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // clusters in tile-fastest order (concurrent clusters spread over tiles);
+    // the CTAs of a cluster take consecutive tasks of the same tile
+    const uint32_t CL = ptx::cluster_nctarank(), rank = ptx::cluster_ctarank();
+    const int64_t n_tiles = (a.N + TN - 1) / TN;
+    const int64_t cluster_id = blockIdx.x / CL;
+    const int task = (int)(cluster_id / n_tiles) * (int)CL + (int)rank;
+    const int64_t n0 = (cluster_id % n_tiles) * TN;
+    const int item_first = task * a.G;
+    const int g_count = task < a.n_tasks ? min(a.G, a.n_items - item_first) : 0;
+    const int C = CT ? CT : a.C;
+    const int nch = a.nchunks;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NS; s++) {
+            ptx::mbar_init(&sh.full[s], 1);
+            ptx::mbar_init(&sh.empty[s], NCW * CL);
+        }
+        ptx::mbar_init(sh.wbar, 1);
+        sh.misc[0] = 0;
+        ptx::fence_barrier_init();
+    }
+    if ((int)threadIdx.x < g_count) {   // one thread per item fills the item table
+        const int g = threadIdx.x;
+        const Item it = a.items[item_first + g];
+        sh.itab[6 * g + 0] = it.row;
+        sh.itab[6 * g + 1] = it.p0;
+        sh.itab[6 * g + 2] = it.p1;
+        sh.itab[6 * g + 3] = it.slot;
+        sh.itab[6 * g + 4] = __ldg(a.rec_off + item_first + g);
+        sh.itab[6 * g + 5] = it.p1 - it.p0;
+    }
+    // every CTA's barriers exist before any multicast or remote arrive
+    if (CL == 1) __syncthreads(); else ptx::cluster_sync();
+
+    if (warp == NCW) {
+        // ---------------- producer: block values by bulk copy, then X chunks
+        if (lane == 0) {
+            ptx::prefetch_tensormap(&xmap);
+            {
+                const int per_block = R * C * WD;
+                uint32_t total = 0;
+                for (int g = 0; g < g_count; g++) {
+                    const int len = sh.itab[6 * g + 5];
+                    total += (uint32_t)xstage_record_ints(len, nch) * 4;
+                    if (a.w_bulk) total += (uint32_t)len * per_block * 4;
+                }
+                ptx::mbar_arrive_expect_tx(sh.wbar, total);
+                int woff = 0, roff = 0;
+                for (int g = 0; g < g_count; g++) {
+                    const int len = sh.itab[6 * g + 5];
+                    const uint32_t wbytes = (uint32_t)len * per_block * 4;
+                    if (a.w_bulk && wbytes)
+                        ptx::bulk_load(sh.W + woff, a.wpk + (int64_t)sh.itab[6 * g + 1] * per_block, wbytes, sh.wbar);
+                    const int rints = (int)xstage_record_ints(len, nch);
+                    ptx::bulk_load(sh.I + roff, a.rec + sh.itab[6 * g + 4], (uint32_t)rints * 4, sh.wbar);
+                    woff += len * per_block;
+                    roff += rints;
+                }
+            }
+            const int rows = TN / (int)CL;                       // this CTA's slice of every chunk
+            const uint16_t mask = (uint16_t)((1u << CL) - 1u);
+            int c = 0;
+            bool ok = true;
+            for (; c < nch; c++) {
+                const int s = c % NS;
+                // the stage is free once every consumer warp of the cluster released it
+                if (c >= NS && !ptx::mbar_wait_cluster_bounded(&sh.empty[s], ((c / NS) - 1) & 1, a.wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                if (aborted(sh.misc)) { ok = false; break; }
+                if (c == a.stall_chunk) continue;   // its consumers time out
+                ptx::mbar_arrive_expect_tx(&sh.full[s], St::kBytes);
+#pragma unroll
+                for (int b = 0; b < St::kBoxes; b++)
+                    ptx::tma_load_2d_multicast(sh.base + s * St::kBytes + b * St::kBoxBytes + rank * rows * 128,
+                                               &xmap, c * KC + b * St::kBoxCols, (int32_t)(n0 + rank * rows),
+                                               &sh.full[s], mask);
+            }
+            if (!ok) {
+                set_status(a.status, DEV_TIMEOUT);
+                atomicExch(&sh.misc[0], 1);
+            }
+            // the last loads issued may still be in flight: wait (bounded) for
+            // them so that no TMA write outlives the CTA
+            for (int d = max(0, c - NS); d < c; d++)
+                if (d != a.stall_chunk) ptx::mbar_wait_bounded(&sh.full[d % NS], (d / NS) & 1, kDrainNs);
+            ptx::mbar_wait_bounded(sh.wbar, 0, kDrainNs);
+        }
+        __syncwarp();
+    } else {
+        consumer<T, TR, NRG, CT>(a, sh, n0, item_first, g_count, CL, warp, lane);
+    }
+    if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
+}
+
+// W^T per block, widened to fp32 (WD copies of each value):
+// wpk[((p*C + c)*R + r)*WD + d] = data[(p*R + r)*C + c].
 template <typename T>
 __global__ void k_pack(const T *__restrict__ data, float *__restrict__ wpk, int64_t nnzb, int R, int C) {
     const int64_t total = nnzb * R * C;
@@ -446,7 +552,9 @@ __global__ void k_pack(const T *__restrict__ data, float *__restrict__ wpk, int6
         const int64_t p = e / ((int64_t)R * C);
         const int rc = (int)(e - p * R * C);
         const int c = rc / R, r = rc - c * R;
-        wpk[e] = to_f32(data[(p * R + r) * C + c]);
+        const float w = to_f32(data[(p * R + r) * C + c]);
+#pragma unroll
+        for (int d = 0; d < WD; d++) wpk[WD * e + d] = w;
     }
 }
 
@@ -469,29 +577,62 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // ring, reused for the epilogue's partial tiles
 size_t region_bytes(bsr_dtype_t dt, int R) {
     const size_t ring = (size_t)NS * (dt == BSR_F32 ? Stage<float>::kBytes : Stage<uint16_t>::kBytes);
-    const size_t part = (size_t)NCW * TN * (R + 4) * 4;
+    const size_t part = (size_t)(NCW * 2 / 3) * TN * (R + 4) * 4;   // most tiles of one tree round (G=4, S=3)
     return (std::max(ring, part) + 1023) & ~size_t(1023);
 }
 
-template <typename T, int TR, int NRG>
+// Whether clusters of CL CTAs with `smem` bytes each can be resident at all
+// (cached per kernel, cluster size, shared-memory size and device).
+bool cluster_fits(const void *func, int CL, uint32_t smem, int dev) {
+    struct Entry {
+        const void *func;
+        int CL, dev;
+        uint32_t smem;
+        bool ok;
+    };
+    static std::mutex mu;
+    static std::vector<Entry> cache;
+    std::lock_guard<std::mutex> lk(mu);
+    for (const Entry &e : cache)
+        if (e.func == func && e.CL == CL && e.smem == smem && e.dev == dev) return e.ok;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)CL);
+    cfg.blockDim = dim3(NTHREADS);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    const bool ok = cudaOccupancyMaxActiveClusters(&n, func, &cfg) == cudaSuccess && n > 0;
+    cudaGetLastError();
+    cache.push_back({func, CL, dev, smem, ok});
+    return ok;
+}
+
+// CTAs per cluster. Multicast only pays where L2 bandwidth, not latency,
+// limits the X stream, so it is opt-in (BSR_XS_CL = 2, 4 or 8).
+int choose_cluster(int n_tasks) {
+    static const int forced = [] {
+        const char *v = getenv("BSR_XS_CL");
+        return v ? atoi(v) : 0;
+    }();
+    if (forced == 2 || forced == 4 || forced == 8) return std::min(forced, std::max(1, n_tasks));
+    return 1;
+}
+
+template <typename T, int TR, int NRG, int CT>
 cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     const Schedule &sc = *la.sc;
     const size_t es = sizeof(T);
     const int gidx = g_index(G);
     const int n_items = (int)sc.items.size();
     if (n_items == 0 || la.N == 0) return cudaSuccess;
-    CUtensorMap map;
     auto enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
-    const cuuint64_t dims[2] = {(cuuint64_t)sc.K, (cuuint64_t)la.N};
-    const cuuint64_t strides[1] = {(cuuint64_t)sc.K * es};
-    const cuuint32_t box[2] = {(cuuint32_t)Stage<T>::kBoxCols, (cuuint32_t)TN};
-    const cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(&map, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                     const_cast<void *>(la.X), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
 
     XsArgs a;
     a.items = sc.d_items;
@@ -499,7 +640,8 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.G = G;
     a.S = NCW / G;
     a.n_tasks = (n_items + G - 1) / G;
-    a.indices = sc.d_indices;
+    a.rec = sc.d_xs_rec;
+    a.rec_off = sc.d_xs_rec_off;
     a.wpk = static_cast<const float *>(la.data);
     a.bias = la.bias;
     a.Y = la.Y;
@@ -512,13 +654,12 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.nchunks = (int)((sc.K + KC - 1) / KC);
     a.w_off = (uint32_t)region_bytes(sc.dt, sc.R);
     a.idx_off = a.w_off + (uint32_t)((pl.task_wbytes[gidx] + 15) & ~size_t(15));
-    a.cb_off = a.idx_off + (uint32_t)((pl.task_ibytes[gidx] + 15) & ~size_t(15));
-    a.bias_off = a.cb_off + (uint32_t)(((size_t)G * (a.nchunks + 1) * 4 + 15) & ~size_t(15));
+    a.bias_off = a.idx_off + (uint32_t)((pl.task_ibytes[gidx] + 15) & ~size_t(15));
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * sc.R * 4 + 15) & ~size_t(15));
-    a.cb = sc.d_xs_cb;
-    a.w_bulk = (sc.R * sc.C) % 4 == 0;
     a.misc_off = a.bar_off + (2 * NS + 1) * 8;
-    const uint32_t smem = a.misc_off + (4 + 6 * 8) * 4 + 1024;   // + slack to align the base
+    // one bulk copy per item needs every item's byte range 16-byte aligned
+    a.w_bulk = (sc.R * sc.C * WD * 4) % 16 == 0;
+    const uint32_t smem = a.misc_off + (4 + 6 * NCW) * 4 + 1024;   // + slack to align the base
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
     static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
@@ -526,28 +667,69 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     cudaGetDevice(&dev);
     const uint64_t bit = 1ull << (dev & 63);
     if (!(attr_set.load() & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kXsMaxSmem);
+        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG, CT>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kXsMaxSmem);
         if (e != cudaSuccess) return e;
         attr_set.fetch_or(bit);
     }
     if (smem > kXsMaxSmem) return cudaErrorInvalidConfiguration;
     const int64_t n_tiles = (la.N + TN - 1) / TN;
-    const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
-    if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-    k_xstage<T, TR, NRG><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
-    return cudaGetLastError();
+
+    cudaError_t err = cudaErrorInvalidConfiguration;
+    for (int CL = choose_cluster(a.n_tasks); CL >= 1; CL >>= 1) {
+        if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT>), CL, smem, dev))
+            continue;
+        const int64_t n_groups = (a.n_tasks + CL - 1) / CL;
+        const int64_t grid = n_tiles * n_groups * CL;   // cluster-major, tile-fastest
+        if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
+        CUtensorMap map;
+        const cuuint64_t dims[2] = {(cuuint64_t)sc.K, (cuuint64_t)la.N};
+        const cuuint64_t strides[1] = {(cuuint64_t)sc.K * es};
+        const cuuint32_t box[2] = {(cuuint32_t)Stage<T>::kBoxCols, (cuuint32_t)(TN / CL)};
+        const cuuint32_t estr[2] = {1, 1};
+        CUresult r = enc(&map, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                         const_cast<void *>(la.X), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+        if (CL == 1) {
+            k_xstage<T, TR, NRG, CT><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
+            err = cudaGetLastError();
+            break;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)grid);
+        cfg.blockDim = dim3(NTHREADS);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = la.stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = (unsigned)CL;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        err = cudaLaunchKernelEx(&cfg, k_xstage<T, TR, NRG, CT>, map, a);
+        break;
+    }
+    return err;
+}
+
+template <typename T, int TR, int NRG>
+cudaError_t launch_c(const LaunchArgs &la, const XsPlan &pl, int G) {
+    if (la.sc->C == 1) return launch_t<T, TR, NRG, 1>(la, pl, G);
+    return launch_t<T, TR, NRG, 0>(la, pl, G);
 }
 
 template <typename T>
 cudaError_t launch_r(const LaunchArgs &la, const XsPlan &pl, int G) {
     switch (la.sc->R) {
-        case 1: return launch_t<T, 1, 1>(la, pl, G);
-        case 2: return launch_t<T, 2, 1>(la, pl, G);
-        case 4: return launch_t<T, 4, 1>(la, pl, G);
-        case 8: return launch_t<T, 8, 1>(la, pl, G);
-        case 16: return launch_t<T, 8, 2>(la, pl, G);
-        case 32: return launch_t<T, 8, 4>(la, pl, G);
+        case 1: return launch_c<T, 1, 1>(la, pl, G);
+        case 2: return launch_c<T, 2, 1>(la, pl, G);
+        case 4: return launch_c<T, 4, 1>(la, pl, G);
+        case 8: return launch_c<T, 8, 1>(la, pl, G);
+        case 16: return launch_c<T, 8, 2>(la, pl, G);
+        case 32: return launch_c<T, 8, 4>(la, pl, G);
     }
     return cudaErrorNotSupported;
 }
@@ -556,17 +738,25 @@ cudaError_t launch_r(const LaunchArgs &la, const XsPlan &pl, int G) {
 
 size_t xstage_smem_bytes(bsr_dtype_t dt, int R, int64_t K, int G, size_t wbytes, size_t ibytes) {
     const size_t nch = (size_t)((K + KC - 1) / KC);
+    (void)nch;
     return region_bytes(dt, R) + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * (nch + 1) * 4 + 15) & ~size_t(15)) + (((size_t)G * R * 4 + 15) & ~size_t(15)) +
-           (2 * NS + 1) * 8 + (4 + 6 * 8) * 4 + 1024;
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + (4 + 6 * NCW) * 4 + 1024;
 }
 
 size_t xstage_task_budget(bsr_dtype_t dt, int R, int64_t K) {
-    const size_t fixed = xstage_smem_bytes(dt, R, K, 8, 0, 0) + 64;
+    const size_t fixed = xstage_smem_bytes(dt, R, K, NCW, 0, 0) + 64;
     return fixed >= (size_t)kXsMaxSmem ? 0 : (size_t)kXsMaxSmem - fixed;
 }
 
-int g_index(int G) { return G == 1 ? 0 : G == 2 ? 1 : G == 4 ? 2 : 3; }
+uint32_t xstage_stage_offset(bsr_dtype_t dt, int kk) {
+    return dt == BSR_F32 ? Stage<float>::off0(kk) : Stage<uint16_t>::off0(kk);
+}
+
+int g_index(int G) {
+    for (int i = 0; i < kXsTaskSizes; i++)
+        if (kXsG[i] == G) return i;
+    return 0;
+}
 
 bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
     const bool r_ok = R == 1 || R == 2 || R == 4 || R == 8 || R == 16 || R == 32;

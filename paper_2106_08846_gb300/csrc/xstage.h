@@ -11,15 +11,36 @@ namespace bsr {
 constexpr int kXsTokens = 64;          // tokens per CTA
 constexpr int kXsChunk = 128;          // K columns per ring stage
 constexpr int kXsStages = 3;           // ring depth
-constexpr int kXsConsumerWarps = 8;
+constexpr int kXsConsumerWarps = 12;   // + 1 producer warp: 16 warps of registers
 constexpr int kXsMaxSmem = 232448;     // 227 KB, the per-CTA opt-in limit
+constexpr int kXsWDup = 1;             // copies of each packed block value
 
-// Per task size G in {1, 2, 4, 8} (index 0..3): the largest shared-memory
-// footprint of block values / indices over all tasks of G consecutive items.
+// Task sizes G (items per CTA); each divides the consumer warps.
+constexpr int kXsTaskSizes = 6;
+constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12};
+
+// Per task size (index into kXsG): the largest shared-memory footprint of
+// block values / indices over all tasks of G consecutive items.
 struct XsPlan {
-    size_t task_wbytes[4] = {0, 0, 0, 0};
-    size_t task_ibytes[4] = {0, 0, 0, 0};
+    size_t task_wbytes[kXsTaskSizes] = {0, 0, 0, 0, 0, 0};
+    size_t task_ibytes[kXsTaskSizes] = {0, 0, 0, 0, 0, 0};   // item records (see xstage_record_ints)
 };
+
+// Per item, the kernel fetches one "record" of int32 by bulk copy:
+//   [ per block: its X offset inside a ring stage (C == 1) or its block
+//     column (C > 1), padded to 4 ints | per K chunk c = 0..nchunks: the
+//     first item-local block of chunk c, padded to 4 ints ]
+#ifdef __CUDACC__
+#define XS_HD __host__ __device__
+#else
+#define XS_HD
+#endif
+XS_HD inline int64_t xstage_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
+XS_HD inline int64_t xstage_record_ints(int64_t len, int64_t nchunks) {
+    return xstage_pad4(len) + xstage_pad4(nchunks + 1);
+}
+// Byte offset of chunk column kk inside a ring stage, token row 0.
+uint32_t xstage_stage_offset(bsr_dtype_t dt, int kk);
 
 int g_index(int G);
 bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K);
