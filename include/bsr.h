@@ -141,6 +141,38 @@ bsr_status_t bsr_check_device_status(bsr_handle_t h);
  */
 bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len);
 
+/*
+ * bsr_spmm_noalloc -- bsr_spmm for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart: this is a deployment aid. Some callers may
+ * not call cudaMalloc at the point where they run the product: code inside
+ * a CUDA graph capture (allocation there is not allowed), code bound to a
+ * fixed memory budget or to its own allocator, and latency-critical loops
+ * where an allocation's implicit device synchronisation is unacceptable.
+ * bsr_spmm allocates when a call needs more split-row workspace than the
+ * handle holds; this entry point never does.
+ *
+ * Same product and arguments as bsr_spmm, except that X and Y must be device
+ * pointers (host buffers would need staging memory: BSR_ERR_INVALID_ARG).
+ * The fp32 partial tiles of block rows that the schedule splits across CTAs
+ * go to one scratch array compiled into the library, of
+ * BSR_NOALLOC_SCRATCH_BYTES bytes, which every GPU that loads the library
+ * holds until the process exits. A call needs slots * N * R * 4 bytes of it
+ * ("slots" and "R" as reported by bsr_get_schedule); a larger call returns
+ * BSR_ERR_CAPACITY and launches nothing.
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current) and keeps it: make that
+ * first call before any stream capture. All calls share the one array, so
+ * calls whose kernels may run at the same time on the GPU (on streams with
+ * no ordering between them) race and produce wrong results. The array keeps
+ * the last call's contents; every element a call reads is written earlier
+ * in the same call, so nothing is cleared.
+ * Calls no cudaMalloc, cudaFree or allocating library routine.
+ */
+#define BSR_NOALLOC_SCRATCH_BYTES (32u << 20)
+bsr_status_t bsr_spmm_noalloc(bsr_handle_t h, const void *X, const float *bias, void *Y, int64_t N,
+                              void *stream);
+
 /* bsr_destroy -- release what the handle owns (not the borrowed arrays). NULL is a no-op. */
 void bsr_destroy(bsr_handle_t h);
 

@@ -61,6 +61,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.bsr_reserve.restype = U
         lib.bsr_spmm.argtypes = [P, P, P, P, I64, P]
         lib.bsr_spmm.restype = U
+        lib.bsr_spmm_noalloc.argtypes = [P, P, P, P, I64, P]
+        lib.bsr_spmm_noalloc.restype = U
         lib.bsr_check_device_status.argtypes = [P]
         lib.bsr_check_device_status.restype = U
         lib.bsr_get_schedule.argtypes = [P, ctypes.c_char_p, ctypes.c_size_t]
@@ -202,6 +204,22 @@ def bsr_spmm(h: Handle, X: torch.Tensor, bias: Optional[torch.Tensor], Y: torch.
     if X.shape[-1] != h.K or Y.shape[-1] != h.M or X.shape[0] < N or Y.shape[0] < N:
         raise ValueError("X must be [N, K] and Y [N, M]")
     _check(load().bsr_spmm(h.ptr, _ptr(X), _ptr(bias), _ptr(Y), N, _stream(stream)), "bsr_spmm")
+
+
+def bsr_spmm_noalloc(h: Handle, X: torch.Tensor, bias: Optional[torch.Tensor], Y: torch.Tensor,
+                     N: Optional[int] = None, stream=None) -> None:
+    """bsr_spmm without any device allocation (device X and Y only): split-row
+    partials use the library's fixed scratch array (see include/bsr.h)."""
+    if X.dtype != h.dtype or Y.dtype != h.dtype:
+        raise TypeError("X and Y must have the handle's dtype")
+    if not X.is_contiguous() or not Y.is_contiguous():
+        raise ValueError("X and Y must be contiguous")
+    if bias is not None and (bias.dtype != torch.float32 or not bias.is_contiguous()):
+        raise TypeError("bias must be a contiguous float32 tensor")
+    N = X.shape[0] if N is None else N
+    if X.shape[-1] != h.K or Y.shape[-1] != h.M or X.shape[0] < N or Y.shape[0] < N:
+        raise ValueError("X must be [N, K] and Y [N, M]")
+    _check(load().bsr_spmm_noalloc(h.ptr, _ptr(X), _ptr(bias), _ptr(Y), N, _stream(stream)), "bsr_spmm_noalloc")
 
 
 def bsr_check_device_status(h: Handle) -> int:
