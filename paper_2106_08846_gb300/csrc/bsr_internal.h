@@ -11,6 +11,7 @@
 #include <vector>
 
 #include "bsr.h"
+#include "tc.h"
 #include "xstage.h"
 
 namespace bsr {
@@ -58,6 +59,7 @@ struct Schedule {
     std::vector<Split> splits;
     std::vector<int32_t> group_begin;   // groups + 1 offsets into items
     XsPlan xs;                          // xstage task footprints
+    TcPlan tc;                          // tcgen05 task footprints
     int n_slots = 0;
     int64_t empty_rows = 0, max_row = 0;
     int sm_count = 148;
@@ -120,6 +122,8 @@ struct LaunchArgs {
 };
 cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
+cudaError_t launch_tc(const LaunchArgs &a, int G);
+cudaError_t pack_tc_data(const void *data, int64_t nnzb, int R, int C, uint16_t *out, cudaStream_t s);
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, float *wpk,
                              cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);

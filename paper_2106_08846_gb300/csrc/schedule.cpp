@@ -76,9 +76,12 @@ int64_t split_limit(const Schedule &sc) {
 
 // For each task size G, the largest block-value and index footprint over
 // the tasks formed by G consecutive items of the (LPT-ordered) item list.
-void plan_xstage(Schedule &sc) {
-    const int64_t nch = (sc.K + kXsChunk - 1) / kXsChunk;
-    // per-item records: block offsets (C == 1) or columns, then chunk starts
+// Per-item records fetched by the kernels: one int per block (`value` of its
+// block column) padded to 4, then the first block of each chunk of `chunk`
+// columns (nchunks + 1 entries) padded to 4.
+template <typename F>
+void build_records(Schedule &sc, int chunk, F value) {
+    const int64_t nch = (sc.K + chunk - 1) / chunk;
     sc.xs_rec.clear();
     sc.xs_rec_off.assign(sc.items.size(), 0);
     for (size_t i = 0; i < sc.items.size(); i++) {
@@ -87,21 +90,24 @@ void plan_xstage(Schedule &sc) {
         sc.xs_rec_off[i] = (int32_t)sc.xs_rec.size();
         const size_t base = sc.xs_rec.size();
         sc.xs_rec.resize(base + (size_t)xstage_record_ints(len, nch), 0);
-        for (int32_t b = 0; b < len; b++) {
-            const int64_t col = sc.indices[it.p0 + b];
-            sc.xs_rec[base + b] = sc.C == 1 ? (int32_t)xstage_stage_offset(sc.dt, (int)(col % kXsChunk)) : (int32_t)col;
-        }
+        for (int32_t b = 0; b < len; b++) sc.xs_rec[base + b] = value((int64_t)sc.indices[it.p0 + b]);
         int32_t b = 0;
         const size_t cbase = base + (size_t)xstage_pad4(len);
         for (int64_t c = 0; c <= nch; c++) {
-            const int64_t first_col = c * (kXsChunk / sc.C);
+            const int64_t first_col = c * (chunk / sc.C);
             while (b < len && sc.indices[it.p0 + b] < first_col) b++;
             sc.xs_rec[cbase + c] = b;
         }
     }
-    const size_t per_block = (size_t)sc.R * sc.C * 4 * kXsWDup;
-    for (int gi = 0; gi < kXsTaskSizes; gi++) {
-        const int G = kXsG[gi];
+}
+
+// For each task size G, the largest block-value and record footprint over
+// the tasks formed by G consecutive items.
+void footprints(const Schedule &sc, size_t per_block, int chunk, const int *Gs, int nG, size_t *wbytes,
+                size_t *ibytes) {
+    const int64_t nch = (sc.K + chunk - 1) / chunk;
+    for (int gi = 0; gi < nG; gi++) {
+        const int G = Gs[gi];
         size_t wmax = 0, imax = 0;
         for (size_t t = 0; t < sc.items.size(); t += G) {
             size_t blocks = 0, rec = 0;
@@ -113,9 +119,23 @@ void plan_xstage(Schedule &sc) {
             wmax = std::max(wmax, blocks * per_block);
             imax = std::max(imax, rec);
         }
-        sc.xs.task_wbytes[gi] = wmax;
-        sc.xs.task_ibytes[gi] = imax;
+        wbytes[gi] = wmax;
+        ibytes[gi] = imax;
     }
+}
+
+void plan_xstage(Schedule &sc) {
+    build_records(sc, kXsChunk, [&](int64_t col) {
+        return sc.C == 1 ? (int32_t)xstage_stage_offset(sc.dt, (int)(col % kXsChunk)) : (int32_t)col;
+    });
+    footprints(sc, (size_t)sc.R * sc.C * 4 * kXsWDup, kXsChunk, kXsG, kXsTaskSizes, sc.xs.task_wbytes,
+               sc.xs.task_ibytes);
+}
+
+void plan_tc(Schedule &sc) {
+    // a block's value: the byte offset of its first column in a 128-byte stage row
+    build_records(sc, kTcChunk, [&](int64_t col) { return (int32_t)(((col * sc.C) % kTcChunk) * 2); });
+    footprints(sc, (size_t)sc.R * sc.C * 2, kTcChunk, kTcG, kTcTaskSizes, sc.tc.task_wbytes, sc.tc.task_ibytes);
 }
 
 const char *env_str(const char *name) {
@@ -136,7 +156,19 @@ bsr_status_t build_schedule(Schedule &sc) {
     }
     const char *force = env_str("BSR_FORCE_VARIANT");
     const bool want_generic = force && std::string(force) == "generic";
-    if (!want_generic && xstage_supports(sc.R, sc.C, sc.dt, sc.K)) {
+    const bool want_xstage = force && std::string(force) == "xstage";
+    if (!want_generic && !want_xstage && tc_supports(sc.R, sc.C, sc.dt, sc.K)) {
+        sc.variant = V_TC;
+        sc.tn = kTcTokens;
+        sc.threads = 192;
+        const int64_t nch = (sc.K + kTcChunk - 1) / kTcChunk;
+        const int64_t avail = (int64_t)tc_task_budget(sc.R) - 4 * xstage_pad4(nch + 1) - 16;
+        const int64_t lmax = std::max<int64_t>(1, avail / (int64_t)((size_t)sc.R * sc.C * 2 + 4));
+        int64_t limit = split_limit(sc);
+        limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
+        make_items(sc, limit);
+        plan_tc(sc);
+    } else if (!want_generic && xstage_supports(sc.R, sc.C, sc.dt, sc.K)) {
         sc.variant = V_XSTAGE;
         sc.tn = kXsTokens;
         sc.threads = (kXsConsumerWarps + 1) * 32;
@@ -168,15 +200,18 @@ bsr_status_t build_schedule(Schedule &sc) {
 bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
     const Schedule &sc = *h.sched;
-    if (sc.variant != V_XSTAGE || sc.nnzb == 0) return BSR_OK;
-    const size_t bytes = (size_t)sc.nnzb * sc.R * sc.C * 4 * kXsWDup;
+    if ((sc.variant != V_XSTAGE && sc.variant != V_TC) || sc.nnzb == 0) return BSR_OK;
+    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * sc.R * sc.C * 2
+                                            : (size_t)sc.nnzb * sc.R * sc.C * 4 * kXsWDup;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
         h.data_packed = nullptr;
         return BSR_ERR_ALLOC;
     }
-    if (pack_xstage_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, (float *)h.data_packed, 0) != cudaSuccess ||
-        cudaDeviceSynchronize() != cudaSuccess) {
+    cudaError_t e = sc.variant == V_TC
+                        ? pack_tc_data(h.data, sc.nnzb, sc.R, sc.C, (uint16_t *)h.data_packed, 0)
+                        : pack_xstage_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, (float *)h.data_packed, 0);
+    if (e != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_CUDA;
     }
@@ -220,9 +255,44 @@ int choose_tasks(const Schedule &sc, int64_t N) {
     return best;
 }
 
+// Task size for the tcgen05 kernel: the same waves x (overhead + work) model,
+// among the G whose accumulators fit tensor memory and whose shared memory fits.
+int choose_tc_tasks(const Schedule &sc, int64_t N) {
+    static const int forced = [] {
+        const char *v = getenv("BSR_TC_G");
+        return v ? atoi(v) : 0;
+    }();
+    auto fits = [&](int G) {
+        const int gi = tc_g_index(G);
+        return G * sc.R <= kTcTmemCols &&
+               tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi]) <= (size_t)kTcMaxSmem;
+    };
+    for (int gi = 0; gi < kTcTaskSizes; gi++)
+        if (forced == kTcG[gi] && fits(forced)) return forced;
+    const double kOverheadItems = 4.0;
+    const int64_t tiles = (N + kTcTokens - 1) / kTcTokens;
+    const int64_t items = (int64_t)sc.items.size();
+    int best = 1;
+    double best_cost = -1.0;
+    for (int gi = 0; gi < kTcTaskSizes; gi++) {
+        const int G = kTcG[gi];
+        if (!fits(G)) continue;
+        const int64_t ctas = tiles * ((items + G - 1) / G);
+        const double waves = (double)((ctas + sc.sm_count - 1) / sc.sm_count);
+        const double cost = waves * (kOverheadItems + (double)std::min<int64_t>(G, items));
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = G;
+        }
+    }
+    return best;
+}
+
 cudaError_t launch_spmm(const LaunchArgs &a) {
     cudaError_t e;
-    if (a.sc->variant == V_XSTAGE)
+    if (a.sc->variant == V_TC)
+        e = launch_tc(a, choose_tc_tasks(*a.sc, a.N));
+    else if (a.sc->variant == V_XSTAGE)
         e = launch_xstage(a, choose_tasks(*a.sc, a.N));
     else
         e = launch_generic(a);

@@ -1,0 +1,452 @@
+// tcgen05 tensor-core BSR x dense kernel for bf16 blocks whose both sides are
+// multiples of 16 ("tc"): every kept block is a dense contraction, so each
+// block of a block row becomes C/16 tcgen05.mma instructions of shape
+// M = 128 tokens, N = R outputs, K = 16, accumulated in fp32 in tensor memory.
+//
+//   warp 0 (one thread)  producer: bulk copies of the task's block values
+//                         (repacked at create time into the MMA's K-major
+//                         core-matrix layout) and item records, then X chunks
+//                         [128 tokens x 64 columns] by 2-D TMA (128-byte
+//                         swizzle) through a 6-stage ring.
+//   warp 1 (one thread)  owns the tensor memory (G * R fp32 columns, one
+//                         block row per R columns) and issues the MMAs: for
+//                         each chunk, the blocks of every item that fall in
+//                         it (first-block tables from the host); a
+//                         tcgen05.commit per chunk releases the stage once
+//                         its MMAs completed.
+//   warps 2..5           epilogue: after the last commit, each reads its 32
+//                         TMEM lanes (tokens), adds the bias, converts to
+//                         bf16 and stores Y (or an fp32 partial for a split
+//                         row).
+//
+// Every wait is bounded by the global timer; a timeout sets the device status
+// word, stops issuing, lets the issued copies and MMAs finish, frees the
+// tensor memory and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <atomic>
+#include <mutex>
+
+#include "bsr_internal.h"
+#include "elem.cuh"
+#include "ptx.cuh"
+#include "tc.h"
+
+namespace bsr {
+
+namespace {
+
+constexpr int TN = kTcTokens;
+constexpr int KC = kTcChunk;
+constexpr int NS = kTcStages;
+constexpr uint32_t kStageBytes = TN * KC * 2;   // 16 KB: 128 rows of 128 bytes
+constexpr int NWARPS = 6;
+constexpr int NTHREADS = NWARPS * 32;
+constexpr uint64_t kDrainNs = 200000000ull;
+
+struct TcArgs {
+    const Item *items;
+    int n_items, G, n_tasks;
+    const int32_t *rec;       // per-item records (as xstage: block values then chunk starts)
+    const int32_t *rec_off;
+    const uint16_t *wpk;      // block values in the MMA's B layout
+    const float *bias;
+    uint16_t *Y;
+    float *ws;
+    int *status;
+    int64_t N, K, M;
+    int C, nchunks;
+    uint32_t w_off, rec_off_smem, bias_off, bar_off, misc_off;
+    uint32_t tmem_cols;
+    uint64_t wait_ns;
+    int stall_chunk;
+};
+
+// ---- tcgen05 / UMMA wrappers
+
+// Shared-memory matrix descriptor: start address, leading and stride byte
+// offsets (16-byte units), descriptor version 1, layout (0: no swizzle,
+// 2: 128-byte swizzle).
+__device__ __forceinline__ uint64_t umma_desc(uint32_t addr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
+    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | (1ull << 46) | ((uint64_t)layout << 61);
+}
+
+// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc));
+}
+
+// The mbarrier arrives once every MMA this thread issued so far completed.
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     ptx::smem_addr(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 lanes x 16 columns of fp32 from tensor memory.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int j = 0; j < 16; j++) v[j] = __uint_as_float(r[j]);
+}
+
+__device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(status, DEV_OK, code); }
+__device__ __forceinline__ bool aborted(const int *flag) { return *reinterpret_cast<const volatile int *>(flag) != 0; }
+
+__device__ __forceinline__ int pad4(int n) { return (n + 3) & ~3; }
+__device__ __forceinline__ int record_ints(int len, int nch) { return pad4(len) + pad4(nch + 1); }
+
+template <int R>
+__global__ void __launch_bounds__(NTHREADS, 1)
+k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *base =
+        reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(base + a.bar_off);
+    uint64_t *empty = full + NS;
+    uint64_t *wbar = empty + NS;
+    uint64_t *done = wbar + 1;
+    int *misc = reinterpret_cast<int *>(base + a.misc_off);   // [0] abort flag, [1] TMEM address
+    int *itab = misc + 4;                                     // per item: row p0 p1 slot rec_off len
+    unsigned char *W_s = base + a.w_off;
+    int32_t *I_s = reinterpret_cast<int32_t *>(base + a.rec_off_smem);
+    float *B_s = reinterpret_cast<float *>(base + a.bias_off);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t n_tiles = (a.N + TN - 1) / TN;
+    const int task = (int)(blockIdx.x / n_tiles);
+    const int64_t n0 = (int64_t)(blockIdx.x % n_tiles) * TN;
+    const int item_first = task * a.G;
+    const int g_count = min(a.G, a.n_items - item_first);
+    const int C = a.C, nch = a.nchunks;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NS; s++) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], 1);
+        }
+        ptx::mbar_init(wbar, 1);
+        ptx::mbar_init(done, 1);
+        misc[0] = 0;
+        ptx::fence_barrier_init();
+    }
+    if ((int)threadIdx.x < g_count) {
+        const int g = threadIdx.x;
+        const Item it = a.items[item_first + g];
+        itab[6 * g + 0] = it.row;
+        itab[6 * g + 1] = it.p0;
+        itab[6 * g + 2] = it.p1;
+        itab[6 * g + 3] = it.slot;
+        itab[6 * g + 4] = __ldg(a.rec_off + item_first + g);
+        itab[6 * g + 5] = it.p1 - it.p0;
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         ptx::smem_addr(&misc[1])),
+                     "r"(a.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = (uint32_t)misc[1];
+
+    if (warp == 0) {
+        // ---------------- producer
+        if (lane == 0) {
+            ptx::prefetch_tensormap(&xmap);
+            const uint32_t wblock = (uint32_t)R * C * 2;
+            uint32_t total = 0;
+            for (int g = 0; g < g_count; g++)
+                total += (uint32_t)itab[6 * g + 5] * wblock + (uint32_t)record_ints(itab[6 * g + 5], nch) * 4;
+            ptx::mbar_arrive_expect_tx(wbar, total);
+            uint32_t woff = 0, roff = 0;
+            for (int g = 0; g < g_count; g++) {
+                const int len = itab[6 * g + 5];
+                if (len) ptx::bulk_load(W_s + woff, a.wpk + (int64_t)itab[6 * g + 1] * R * C, len * wblock, wbar);
+                const int rints = record_ints(len, nch);
+                ptx::bulk_load(I_s + roff, a.rec + itab[6 * g + 4], (uint32_t)rints * 4, wbar);
+                woff += len * wblock;
+                roff += rints;
+            }
+            int c = 0;
+            bool ok = true;
+            for (; c < nch; c++) {
+                const int s = c % NS;
+                if (c >= NS && !ptx::mbar_wait_bounded(&empty[s], ((c / NS) - 1) & 1, a.wait_ns)) {
+                    ok = false;
+                    break;
+                }
+                if (aborted(misc)) { ok = false; break; }
+                if (c == a.stall_chunk) continue;   // test hook: its consumer times out
+                ptx::mbar_arrive_expect_tx(&full[s], kStageBytes);
+                ptx::tma_load_2d(base + s * kStageBytes, &xmap, c * KC, (int32_t)n0, &full[s]);
+            }
+            if (!ok) {
+                set_status(a.status, DEV_TIMEOUT);
+                atomicExch(&misc[0], 1);
+            }
+            for (int d = max(0, c - NS); d < c; d++)
+                if (d != a.stall_chunk) ptx::mbar_wait_bounded(&full[d % NS], (d / NS) & 1, kDrainNs);
+            ptx::mbar_wait_bounded(wbar, 0, kDrainNs);
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16(TN, R);
+            bool ok = ptx::mbar_wait_bounded(wbar, 0, a.wait_ns) && !aborted(misc);
+            const uint32_t w_base = ptx::smem_addr(W_s);
+            uint32_t started = 0;
+            for (int c = 0; ok && c < nch; c++) {
+                const int s = c % NS;
+                if (!ptx::mbar_wait_bounded(&full[s], (c / NS) & 1, a.wait_ns) || aborted(misc)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t stage = ptx::smem_addr(base + s * kStageBytes);
+                int wblocks = 0, roff = 0;
+                for (int g = 0; g < g_count; g++) {
+                    const int len = itab[6 * g + 5];
+                    const int32_t *rec = I_s + roff;
+                    const int32_t *cb = rec + pad4(len);
+                    for (int b = cb[c]; b < cb[c + 1]; b++) {
+                        const uint32_t a_row = stage + (uint32_t)rec[b];   // byte offset of the block's columns
+                        const uint32_t w_blk = w_base + (uint32_t)(wblocks + b) * (R * C * 2);
+                        for (int sl = 0; sl < C / 16; sl++) {
+                            const uint64_t ad = umma_desc(a_row + sl * 32, 16, 1024, 2);
+                            const uint64_t bd = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
+                            mma_bf16(tmem + g * R, ad, bd, idesc, ((started >> g) & 1u) | (sl > 0));
+                            started |= 1u << g;
+                        }
+                    }
+                    wblocks += len;
+                    roff += record_ints(len, nch);
+                }
+                mma_commit(&empty[s]);   // the stage is free once these MMAs completed
+            }
+            if (!ok) {
+                set_status(a.status, DEV_TIMEOUT);
+                atomicExch(&misc[0], 1);
+            }
+            mma_commit(done);   // every MMA issued above completes before `done`
+        }
+    } else {
+        // ---------------- epilogue: warps 2..5, TMEM lane quarter = warp % 4
+        const int et = threadIdx.x - 64;   // 0..127
+        for (int e = et; e < g_count * R; e += 128) {
+            const int g = e / R, r = e - g * R;
+            B_s[e] = a.bias ? __ldg(a.bias + (int64_t)itab[6 * g + 0] * R + r) : 0.f;
+        }
+        ptx::named_barrier(1, 128);
+        // the last commit fires after the whole main loop: allow it every chunk's bound
+        const uint64_t limit = a.wait_ns * (uint64_t)(nch + 2);
+        const bool got = ptx::mbar_wait_bounded(done, 0, limit);
+        tc_fence_after();
+        const bool stop = ptx::named_barrier_or(1, 128, !got || aborted(misc));
+        if (!got && et == 0) set_status(a.status, DEV_TIMEOUT);
+        const int q = warp & 3;
+        const int64_t n = n0 + 32 * q + lane;
+        for (int g = 0; g < g_count && !stop; g++) {
+            const int len = itab[6 * g + 5], row = itab[6 * g + 0], slot = itab[6 * g + 3];
+#pragma unroll
+            for (int h = 0; h < R; h += 16) {
+                float v[16];
+                if (len > 0) {
+                    tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(g * R + h), v);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 16; j++) v[j] = 0.f;
+                }
+                if (n >= a.N) continue;
+                if (slot < 0) {
+                    uint32_t pk[8];
+#pragma unroll
+                    for (int j = 0; j < 8; j++) {
+                        const float lo = v[2 * j] + B_s[g * R + h + 2 * j];
+                        const float hi = v[2 * j + 1] + B_s[g * R + h + 2 * j + 1];
+                        pk[j] = (uint32_t)from_f32<uint16_t>(lo) | ((uint32_t)from_f32<uint16_t>(hi) << 16);
+                    }
+                    uint4 *dst = reinterpret_cast<uint4 *>(a.Y + n * a.M + (int64_t)row * R + h);
+                    dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                    dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                } else {
+                    float4 *dst = reinterpret_cast<float4 *>(a.ws + ((int64_t)slot * a.N + n) * R + h);
+#pragma unroll
+                    for (int j = 0; j < 4; j++) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                }
+            }
+        }
+    }
+    // ---------------- teardown: every MMA completed (the epilogue waited for
+    // `done`, or the issuer never started), then free the tensor memory
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(a.tmem_cols) : "memory");
+    }
+}
+
+// Block values into the MMA's B operand layout (K-major, no swizzle): for each
+// K-slice of 16 columns, 8-row x 16-byte core matrices, 128 bytes apart along
+// K and 256 bytes apart along the rows.
+__global__ void k_pack_tc(const uint16_t *__restrict__ data, uint16_t *__restrict__ out, int64_t nnzb, int R, int C) {
+    const int64_t total = nnzb * R * C;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = e / ((int64_t)R * C);
+        const int rc = (int)(e - p * R * C);
+        const int n = rc / C, k = rc - n * C;
+        const int64_t dst = p * R * C + (k >> 4) * (R * 16) + (n >> 3) * 128 + ((k & 15) >> 3) * 64 + (n & 7) * 8 + (k & 7);
+        out[dst] = data[e];
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        else
+            cudaGetLastError();
+    });
+    return fn;
+}
+
+uint32_t tmem_cols_for(int cols) {
+    uint32_t n = 32;
+    while ((int)n < cols) n <<= 1;
+    return n;
+}
+
+template <int R>
+cudaError_t launch_r(const LaunchArgs &la, int G) {
+    const Schedule &sc = *la.sc;
+    const int n_items = (int)sc.items.size();
+    if (n_items == 0 || la.N == 0) return cudaSuccess;
+    auto enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    const int gidx = tc_g_index(G);
+    TcArgs a;
+    a.items = sc.d_items;
+    a.n_items = n_items;
+    a.G = G;
+    a.n_tasks = (n_items + G - 1) / G;
+    a.rec = sc.d_xs_rec;
+    a.rec_off = sc.d_xs_rec_off;
+    a.wpk = static_cast<const uint16_t *>(la.data);
+    a.bias = la.bias;
+    a.Y = static_cast<uint16_t *>(la.Y);
+    a.ws = la.ws;
+    a.status = la.status;
+    a.N = la.N;
+    a.K = sc.K;
+    a.M = sc.M;
+    a.C = sc.C;
+    a.nchunks = (int)((sc.K + KC - 1) / KC);
+    a.w_off = NS * kStageBytes;
+    a.rec_off_smem = a.w_off + (uint32_t)((sc.tc.task_wbytes[gidx] + 15) & ~size_t(15));
+    a.bias_off = a.rec_off_smem + (uint32_t)((sc.tc.task_ibytes[gidx] + 15) & ~size_t(15));
+    a.bar_off = a.bias_off + (uint32_t)(((size_t)G * R * 4 + 15) & ~size_t(15));
+    a.misc_off = a.bar_off + (2 * NS + 2) * 8;
+    a.tmem_cols = tmem_cols_for(G * R);
+    a.wait_ns = la.wait_ns;
+    a.stall_chunk = la.stall_chunk;
+    const uint32_t smem = a.misc_off + (4 + 6 * 32) * 4 + 1024;
+    if (smem > (uint32_t)kTcMaxSmem || G * R > kTcTmemCols) return cudaErrorInvalidConfiguration;
+    static std::atomic<uint64_t> attr_set{0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    const uint64_t bit = 1ull << (dev & 63);
+    if (!(attr_set.load() & bit)) {
+        cudaError_t e = cudaFuncSetAttribute(k_tc<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem);
+        if (e != cudaSuccess) return e;
+        attr_set.fetch_or(bit);
+    }
+    CUtensorMap map;
+    const cuuint64_t dims[2] = {(cuuint64_t)sc.K, (cuuint64_t)la.N};
+    const cuuint64_t strides[1] = {(cuuint64_t)sc.K * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)KC, (cuuint32_t)TN};
+    const cuuint32_t estr[2] = {1, 1};
+    if (enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(la.X), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    const int64_t n_tiles = (la.N + TN - 1) / TN;
+    const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
+    if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
+    k_tc<R><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
+    const bool r_ok = R == 16 || R == 32 || R == 64 || R == 128;
+    const bool c_ok = C == 16 || C == 32 || C == 64;
+    return dt == BSR_BF16 && r_ok && c_ok && K % 8 == 0 && K > 0;
+}
+
+int tc_g_index(int G) {
+    for (int i = 0; i < kTcTaskSizes; i++)
+        if (kTcG[i] == G) return i;
+    return 0;
+}
+
+size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes) {
+    return (size_t)NS * kStageBytes + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 2) * 8 + (4 + 6 * 32) * 4 + 1024;
+}
+
+size_t tc_task_budget(int R) {
+    const size_t fixed = tc_smem_bytes(R, 32, 0, 0) + 64;
+    return fixed >= (size_t)kTcMaxSmem ? 0 : (size_t)kTcMaxSmem - fixed;
+}
+
+uint32_t tc_block_offset(int kk) { return (uint32_t)kk * 2; }
+
+cudaError_t pack_tc_data(const void *data, int64_t nnzb, int R, int C, uint16_t *out, cudaStream_t s) {
+    const int64_t total = nnzb * R * C;
+    if (total == 0) return cudaSuccess;
+    const int grid = (int)std::min<int64_t>((total + 255) / 256, 1 << 20);
+    k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), out, nnzb, R, C);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tc(const LaunchArgs &la, int G) {
+    switch (la.sc->R) {
+        case 16: return launch_r<16>(la, G);
+        case 32: return launch_r<32>(la, G);
+        case 64: return launch_r<64>(la, G);
+        case 128: return launch_r<128>(la, G);
+    }
+    return cudaErrorNotSupported;
+}
+
+}  // namespace bsr

@@ -270,26 +270,36 @@ def test_error_statuses():
     assert h.check_device_status() == b.BSR_OK
 
 
-def test_bounded_wait_times_out_and_reports(monkeypatch):
+@pytest.mark.parametrize("R,C,dtype,variant", [(32, 1, "f32", "xstage"), (16, 16, "bf16", "tcgen05")])
+def test_bounded_wait_times_out_and_reports(monkeypatch, R, C, dtype, variant):
     """An X chunk that is never loaded: every wait on it gives up after the
-    bound (2 ms here), the kernel records BSR_ERR_TIMEOUT and returns; the
-    context stays usable and a normal handle still computes correctly."""
+    bound (2 ms here), the kernel records BSR_ERR_TIMEOUT, releases what it
+    holds and returns; the context stays usable and a normal handle still
+    computes correctly."""
     bsr = _bsr()
     from paper_2106_08846_gb300 import bsrlib as b
-    w = _weight(256, 512, 32, 1, "f32", 0.2, 21)
-    gpu = build_on_gpu(w.W, 32, 1)
+    w = _weight(256, 512, R, C, dtype, 0.2, 21)
+    gpu = build_on_gpu(w.W, R, C)
     monkeypatch.setenv("BSR_WAIT_LIMIT_NS", "2000000")
     monkeypatch.setenv("BSR_TEST_STALL_CHUNK", "1")
-    h = bsr.bsr_create(*gpu, 32, 1, 256, 512)
+    h = bsr.bsr_create(*gpu, R, C, 256, 512)
     monkeypatch.delenv("BSR_WAIT_LIMIT_NS")
     monkeypatch.delenv("BSR_TEST_STALL_CHUNK")
-    if h.schedule()["variant"] != "xstage":
-        pytest.skip("no bounded wait on this path")
-    X = synth.activations(22, 128, 512, "f32")
+    assert h.schedule()["variant"] == variant
+    X = synth.activations(22, 128, 512, dtype)
     h.spmm(to_dev(X), to_dev(w.bias))
     assert h.check_device_status() == b.BSR_ERR_TIMEOUT
     assert h.check_device_status() == b.BSR_OK          # cleared after reading
-    h2 = bsr.bsr_create(*gpu, 32, 1, 256, 512)
+    h2 = bsr.bsr_create(*gpu, R, C, 256, 512)
     Y = to_host(h2.spmm(to_dev(X), to_dev(w.bias)))
     assert h2.check_device_status() == b.BSR_OK
-    check_product(Y, oracle.bsr_from_dense(w.W, 32, 1), X, w.bias, 256)
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, 256)
+
+
+@pytest.mark.parametrize("R,C", [(16, 16), (32, 32), (64, 64), (16, 32), (32, 16)])
+def test_tensor_core_path_is_used_for_bf16_square_blocks(R, C):
+    w = _weight(256, 512, R, C, "bf16", 0.25, 30 + R + C)
+    X = synth.activations(31, 200, 512, "bf16")
+    h, _, Y = _run(w, X)
+    assert h.schedule()["variant"] == "tcgen05"
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, 256)
