@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer pass (profiling runs)")
+    ap.add_argument("--shapes", default="", help="comma-separated subset of block shapes, e.g. 1x1,32x1 (profiling runs)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
 
@@ -226,6 +228,37 @@ def run_reference(args, world, rank):
 
 # ------------------------------------------------------------------ GPU arm
 
+def run_e2e(bsr, handles, biases, wl, X_np, N, K, stream, world, flops_step):
+    """The step through the C ABI with pinned host X and Y: each call copies X
+    in and Y out on the stream (inside the call), so the copies are timed."""
+    import torch
+    Xh = torch.from_numpy(X_np).pin_memory()
+    Yh = [torch.empty((N, w.M), dtype=torch.float32).pin_memory() for w in wl.weights]
+    for h, Y in zip(handles, Yh):
+        bsr.bsr_spmm(h, Xh, None, Y, N, stream)       # sizes the staging buffers
+    torch.cuda.synchronize()
+
+    def e2e_step():
+        for h, b, Y in zip(handles, biases, Yh):
+            bsr.bsr_spmm(h, Xh, b, Y, N, stream)
+
+    for _ in range(3):
+        e2e_step()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+    value = world * flops_step * K / (e2e_ms * 1e-3) / 1e9
+    h2d = sum(N * w.K * 4 for w in wl.weights)
+    d2h = sum(N * w.M * 4 for w in wl.weights)
+    return value, h2d, d2h
+
+
 def run_ours(args, world, rank, local):
     import torch
 
@@ -241,6 +274,9 @@ def run_ours(args, world, rank, local):
     bsr.load()
 
     wl = synth.config(2)
+    if args.shapes:
+        keep = set(args.shapes.split(","))
+        wl.weights = [w for w in wl.weights if f"{w.R}x{w.C}" in keep]
     N = wl.N
     X_np = wl.make_X()
     X = torch.from_numpy(X_np).to(dev)
@@ -305,30 +341,11 @@ def run_ours(args, world, rank, local):
     gbs = world * sum(nbytes) * K / (total_ms * 1e-3) / 1e9
 
     # ---- e2e: pinned host X and Y through the C ABI (copies inside the call)
-    Xh = torch.from_numpy(X_np).pin_memory()
-    Yh = [torch.empty((N, w.M), dtype=torch.float32).pin_memory() for w in wl.weights]
-    for h, Y in zip(handles, Yh):
-        bsr.bsr_spmm(h, Xh, None, Y, N, stream)       # sizes the staging buffers
-    torch.cuda.synchronize()
-
-    def e2e_step():
-        for h, b, Y in zip(handles, biases, Yh):
-            bsr.bsr_spmm(h, Xh, b, Y, N, stream)
-
-    for _ in range(3):
-        e2e_step()
-    torch.cuda.synchronize()
-    barrier(world)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(K):
-        e2e_step()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
-    e2e_value = world * flops_step * K / (e2e_ms * 1e-3) / 1e9
-    h2d = sum(N * w.K * 4 for w in wl.weights)
-    d2h = sum(N * w.M * 4 for w in wl.weights)
+    e2e_value = None
+    if not args.no_e2e:
+        e2e_value, h2d, d2h = run_e2e(bsr, handles, biases, wl, X_np, N, K, stream, world, flops_step)
+    else:
+        h2d = d2h = 0
 
     # ---- dominant kernel vs its roofline
     shares = [kern_ms[i] for i in range(nshape)]
@@ -373,7 +390,8 @@ def run_ours(args, world, rank, local):
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"},
             "gbs": gbs, "gpu_launches": launches_per_step * K,
             "clocks": clocks.summary(),
-            "e2e": {"value": e2e_value, "unit": "GFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "e2e": ({"value": e2e_value, "unit": "GFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+                    if e2e_value is not None else None),
             "roofline": roofline,
             "cpu_baseline": cpu,
             "per_shape": per_shape,

@@ -119,6 +119,10 @@ Schedule::~Schedule() {
     cudaFree(d_indptr);
     cudaFree(d_xs_rec);
     cudaFree(d_xs_rec_off);
+    for (int gi = 0; gi < kTcTaskSizes; gi++) {
+        cudaFree(tc.d_rec[gi]);
+        cudaFree(tc.d_rec_off[gi]);
+    }
     cudaFree(d_indices);
 }
 

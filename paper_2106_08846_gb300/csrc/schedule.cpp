@@ -133,9 +133,48 @@ void plan_xstage(Schedule &sc) {
 }
 
 void plan_tc(Schedule &sc) {
-    // a block's value: the byte offset of its first column in a 128-byte stage row
-    build_records(sc, kTcChunk, [&](int64_t col) { return (int32_t)(((col * sc.C) % kTcChunk) * 2); });
-    footprints(sc, (size_t)sc.R * sc.C * 2, kTcChunk, kTcG, kTcTaskSizes, sc.tc.task_wbytes, sc.tc.task_ibytes);
+    const int64_t nch = (sc.K + kTcChunk - 1) / kTcChunk;
+    const size_t per_block = (size_t)sc.R * sc.C * 2;
+    for (int gi = 0; gi < kTcTaskSizes; gi++) {
+        const int G = kTcG[gi];
+        std::vector<int32_t> &rec = sc.tc.rec[gi];
+        std::vector<int32_t> &off = sc.tc.rec_off[gi];
+        rec.clear();
+        off.clear();
+        size_t wmax = 0, imax = 0;
+        std::vector<std::vector<int32_t>> per_chunk((size_t)nch);
+        for (size_t t = 0; t < sc.items.size(); t += G) {
+            for (auto &v : per_chunk) v.clear();
+            int32_t wblk = 0;
+            const size_t t_end = std::min(sc.items.size(), t + G);
+            for (size_t k = t; k < t_end; k++) {
+                const Item &it = sc.items[k];
+                for (int32_t b = 0; b < it.p1 - it.p0; b++) {
+                    const int64_t col = sc.indices[it.p0 + b];
+                    const int64_t c = (col * sc.C) / kTcChunk;
+                    const int32_t a32 = (int32_t)(((col * sc.C) % kTcChunk) * 2 / 32);
+                    per_chunk[(size_t)c].push_back(a32 | (int32_t)((k - t) << 2) | ((b == 0) << 7) |
+                                                   ((wblk + b) << 8));
+                }
+                wblk += it.p1 - it.p0;
+            }
+            off.push_back((int32_t)rec.size());
+            const size_t head = rec.size();
+            rec.resize(head + (size_t)tc_pad4(nch + 1), 0);
+            int32_t n = 0;
+            for (int64_t c = 0; c < nch; c++) {
+                rec[head + (size_t)c] = n;
+                n += (int32_t)per_chunk[(size_t)c].size();
+            }
+            rec[head + (size_t)nch] = n;
+            for (int64_t c = 0; c < nch; c++) rec.insert(rec.end(), per_chunk[(size_t)c].begin(), per_chunk[(size_t)c].end());
+            rec.resize(head + (size_t)tc_pad4(nch + 1) + (size_t)tc_pad4(n), 0);
+            wmax = std::max(wmax, (size_t)wblk * per_block);
+            imax = std::max(imax, (rec.size() - head) * 4);
+        }
+        sc.tc.task_wbytes[gi] = wmax;
+        sc.tc.task_ibytes[gi] = imax;
+    }
 }
 
 const char *env_str(const char *name) {
@@ -194,6 +233,12 @@ bsr_status_t build_schedule(Schedule &sc) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
+    for (int gi = 0; gi < kTcTaskSizes; gi++)
+        if (upload(&sc.tc.d_rec[gi], sc.tc.rec[gi]) != cudaSuccess ||
+            upload(&sc.tc.d_rec_off[gi], sc.tc.rec_off[gi]) != cudaSuccess) {
+            cudaGetLastError();
+            return BSR_ERR_ALLOC;
+        }
     return BSR_OK;
 }
 

@@ -9,11 +9,12 @@
 //                         [128 tokens x 64 columns] by 2-D TMA (128-byte
 //                         swizzle) through a 6-stage ring.
 //   warp 1 (one thread)  owns the tensor memory (G * R fp32 columns, one
-//                         block row per R columns) and issues the MMAs: for
-//                         each chunk, the blocks of every item that fall in
-//                         it (first-block tables from the host); a
-//                         tcgen05.commit per chunk releases the stage once
-//                         its MMAs completed.
+//                         block row per R columns) and issues the MMAs from
+//                         the task's work list (built on the host): per K
+//                         chunk, one entry per block of any of the task's
+//                         items in it. Chunks without entries are neither
+//                         loaded nor visited. A tcgen05.commit per chunk
+//                         releases the stage once its MMAs completed.
 //   warps 2..5           epilogue: after the last commit, each reads its 32
 //                         TMEM lanes (tokens), adds the bias, converts to
 //                         bf16 and stores Y (or an fp32 partial for a split
@@ -49,8 +50,8 @@ constexpr uint64_t kDrainNs = 200000000ull;
 struct TcArgs {
     const Item *items;
     int n_items, G, n_tasks;
-    const int32_t *rec;       // per-item records (as xstage: block values then chunk starts)
-    const int32_t *rec_off;
+    const int32_t *trec;      // task records: chunk starts, then MMA entries
+    const int32_t *trec_off;  // per task: record offset (ints)
     const uint16_t *wpk;      // block values in the MMA's B layout
     const float *bias;
     uint16_t *Y;
@@ -58,7 +59,7 @@ struct TcArgs {
     int *status;
     int64_t N, K, M;
     int C, nchunks;
-    uint32_t w_off, rec_off_smem, bias_off, bar_off, misc_off;
+    uint32_t w_off, trec_smem, bias_off, bar_off, misc_off;
     uint32_t tmem_cols;
     uint64_t wait_ns;
     int stall_chunk;
@@ -113,7 +114,18 @@ __device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(st
 __device__ __forceinline__ bool aborted(const int *flag) { return *reinterpret_cast<const volatile int *>(flag) != 0; }
 
 __device__ __forceinline__ int pad4(int n) { return (n + 3) & ~3; }
-__device__ __forceinline__ int record_ints(int len, int nch) { return pad4(len) + pad4(nch + 1); }
+
+// 32 lanes x 32 columns of fp32 from tensor memory (no wait).
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
 
 template <int R>
 __global__ void __launch_bounds__(NTHREADS, 1)
@@ -123,12 +135,13 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(base + a.bar_off);
     uint64_t *empty = full + NS;
-    uint64_t *wbar = empty + NS;
-    uint64_t *done = wbar + 1;
+    uint64_t *wbar = empty + NS;     // block values landed
+    uint64_t *done = wbar + 1;       // every MMA completed
+    uint64_t *rbar = done + 1;       // task record landed
     int *misc = reinterpret_cast<int *>(base + a.misc_off);   // [0] abort flag, [1] TMEM address
-    int *itab = misc + 4;                                     // per item: row p0 p1 slot rec_off len
+    int *itab = misc + 4;                                     // per item: row p0 p1 slot - len
     unsigned char *W_s = base + a.w_off;
-    int32_t *I_s = reinterpret_cast<int32_t *>(base + a.rec_off_smem);
+    int32_t *I_s = reinterpret_cast<int32_t *>(base + a.trec_smem);   // the task record
     float *B_s = reinterpret_cast<float *>(base + a.bias_off);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -146,6 +159,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         }
         ptx::mbar_init(wbar, 1);
         ptx::mbar_init(done, 1);
+        ptx::mbar_init(rbar, 1);
         misc[0] = 0;
         ptx::fence_barrier_init();
     }
@@ -156,7 +170,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         itab[6 * g + 1] = it.p0;
         itab[6 * g + 2] = it.p1;
         itab[6 * g + 3] = it.slot;
-        itab[6 * g + 4] = __ldg(a.rec_off + item_first + g);
+        itab[6 * g + 4] = 0;
         itab[6 * g + 5] = it.p1 - it.p0;
     }
     if (warp == 1) {
@@ -175,75 +189,82 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         // ---------------- producer
         if (lane == 0) {
             ptx::prefetch_tensormap(&xmap);
+            const int32_t *trec = a.trec + __ldg(a.trec_off + task);
+            const int n_ent = __ldg(trec + nch);
+            const uint32_t rec_bytes = (uint32_t)(pad4(nch + 1) + pad4(n_ent)) * 4;
+            ptx::mbar_arrive_expect_tx(rbar, rec_bytes);
+            ptx::bulk_load(I_s, trec, rec_bytes, rbar);
             const uint32_t wblock = (uint32_t)R * C * 2;
             uint32_t total = 0;
-            for (int g = 0; g < g_count; g++)
-                total += (uint32_t)itab[6 * g + 5] * wblock + (uint32_t)record_ints(itab[6 * g + 5], nch) * 4;
+            for (int g = 0; g < g_count; g++) total += (uint32_t)itab[6 * g + 5] * wblock;
             ptx::mbar_arrive_expect_tx(wbar, total);
-            uint32_t woff = 0, roff = 0;
+            uint32_t woff = 0;
             for (int g = 0; g < g_count; g++) {
                 const int len = itab[6 * g + 5];
                 if (len) ptx::bulk_load(W_s + woff, a.wpk + (int64_t)itab[6 * g + 1] * R * C, len * wblock, wbar);
-                const int rints = record_ints(len, nch);
-                ptx::bulk_load(I_s + roff, a.rec + itab[6 * g + 4], (uint32_t)rints * 4, wbar);
                 woff += len * wblock;
-                roff += rints;
             }
-            int c = 0;
-            bool ok = true;
-            for (; c < nch; c++) {
-                const int s = c % NS;
-                if (c >= NS && !ptx::mbar_wait_bounded(&empty[s], ((c / NS) - 1) & 1, a.wait_ns)) {
+            int k = 0;          // ring slots used (chunks with work, in order)
+            int stalled = -1;   // test hook: the slot left empty
+            bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);   // chunk starts, from shared memory
+            for (int c = 0; ok && c < nch; c++) {
+                if (I_s[c] == I_s[c + 1]) continue;   // no block of this task in chunk c
+                const int s = k % NS;
+                if (k >= NS && !ptx::mbar_wait_bounded(&empty[s], ((k / NS) - 1) & 1, a.wait_ns)) {
                     ok = false;
                     break;
                 }
                 if (aborted(misc)) { ok = false; break; }
-                if (c == a.stall_chunk) continue;   // test hook: its consumer times out
+                if (c == a.stall_chunk) {   // never loaded: its consumer times out
+                    stalled = k++;
+                    continue;
+                }
                 ptx::mbar_arrive_expect_tx(&full[s], kStageBytes);
                 ptx::tma_load_2d(base + s * kStageBytes, &xmap, c * KC, (int32_t)n0, &full[s]);
+                k++;
             }
             if (!ok) {
                 set_status(a.status, DEV_TIMEOUT);
                 atomicExch(&misc[0], 1);
             }
-            for (int d = max(0, c - NS); d < c; d++)
-                if (d != a.stall_chunk) ptx::mbar_wait_bounded(&full[d % NS], (d / NS) & 1, kDrainNs);
+            for (int d = max(0, k - NS); d < k; d++)
+                if (d != stalled) ptx::mbar_wait_bounded(&full[d % NS], (d / NS) & 1, kDrainNs);
             ptx::mbar_wait_bounded(wbar, 0, kDrainNs);
+            ptx::mbar_wait_bounded(rbar, 0, kDrainNs);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = idesc_bf16(TN, R);
-            bool ok = ptx::mbar_wait_bounded(wbar, 0, a.wait_ns) && !aborted(misc);
+            bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns) && ptx::mbar_wait_bounded(wbar, 0, a.wait_ns) &&
+                      !aborted(misc);
             const uint32_t w_base = ptx::smem_addr(W_s);
-            uint32_t started = 0;
+            const int32_t *ent = I_s + pad4(nch + 1);
+            int k = 0;   // chunks consumed
             for (int c = 0; ok && c < nch; c++) {
-                const int s = c % NS;
-                if (!ptx::mbar_wait_bounded(&full[s], (c / NS) & 1, a.wait_ns) || aborted(misc)) {
+                const int lo = I_s[c], hi = I_s[c + 1];
+                if (lo == hi) continue;
+                const int s = k % NS;
+                if (!ptx::mbar_wait_bounded(&full[s], (k / NS) & 1, a.wait_ns) || aborted(misc)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 const uint32_t stage = ptx::smem_addr(base + s * kStageBytes);
-                int wblocks = 0, roff = 0;
-                for (int g = 0; g < g_count; g++) {
-                    const int len = itab[6 * g + 5];
-                    const int32_t *rec = I_s + roff;
-                    const int32_t *cb = rec + pad4(len);
-                    for (int b = cb[c]; b < cb[c + 1]; b++) {
-                        const uint32_t a_row = stage + (uint32_t)rec[b];   // byte offset of the block's columns
-                        const uint32_t w_blk = w_base + (uint32_t)(wblocks + b) * (R * C * 2);
-                        for (int sl = 0; sl < C / 16; sl++) {
-                            const uint64_t ad = umma_desc(a_row + sl * 32, 16, 1024, 2);
-                            const uint64_t bd = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
-                            mma_bf16(tmem + g * R, ad, bd, idesc, ((started >> g) & 1u) | (sl > 0));
-                            started |= 1u << g;
-                        }
+                for (int e = lo; e < hi; e++) {
+                    const uint32_t v = (uint32_t)ent[e];
+                    const uint32_t a_row = stage + (v & 3u) * 32u;
+                    const uint32_t g = (v >> 2) & 31u, first = (v >> 7) & 1u;
+                    const uint32_t w_blk = w_base + (v >> 8) * (uint32_t)(R * C * 2);
+#pragma unroll 4
+                    for (int sl = 0; sl < C / 16; sl++) {
+                        const uint64_t ad = umma_desc(a_row + sl * 32, 16, 1024, 2);
+                        const uint64_t bd = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
+                        mma_bf16(tmem + g * R, ad, bd, idesc, (first == 0u) | (sl > 0));
                     }
-                    wblocks += len;
-                    roff += record_ints(len, nch);
                 }
                 mma_commit(&empty[s]);   // the stage is free once these MMAs completed
+                k++;
             }
             if (!ok) {
                 set_status(a.status, DEV_TIMEOUT);
@@ -267,31 +288,36 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         if (!got && et == 0) set_status(a.status, DEV_TIMEOUT);
         const int q = warp & 3;
         const int64_t n = n0 + 32 * q + lane;
-        for (int g = 0; g < g_count && !stop; g++) {
-            const int len = itab[6 * g + 5], row = itab[6 * g + 0], slot = itab[6 * g + 3];
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16);
+        // 64 accumulator columns per round: two loads in flight, one wait
+        for (int c0 = 0; c0 < g_count * R && !stop; c0 += 64) {
+            uint32_t r0[32], r1[32];
+            tmem_ld32_nowait(lane_base + c0, r0);
+            if (c0 + 32 < g_count * R) tmem_ld32_nowait(lane_base + c0 + 32, r1);
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            if (n >= a.N) continue;
 #pragma unroll
-            for (int h = 0; h < R; h += 16) {
+            for (int h = 0; h < 64; h += 16) {
+                const int col = c0 + h;
+                if (col >= g_count * R) break;
+                const int g = col / R, hr = col - g * R;
+                const int len = itab[6 * g + 5], row = itab[6 * g + 0], slot = itab[6 * g + 3];
                 float v[16];
-                if (len > 0) {
-                    tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(g * R + h), v);
-                } else {
 #pragma unroll
-                    for (int j = 0; j < 16; j++) v[j] = 0.f;
-                }
-                if (n >= a.N) continue;
+                for (int j = 0; j < 16; j++) v[j] = len > 0 ? __uint_as_float(h < 32 ? r0[h + j] : r1[h - 32 + j]) : 0.f;
                 if (slot < 0) {
                     uint32_t pk[8];
 #pragma unroll
                     for (int j = 0; j < 8; j++) {
-                        const float lo = v[2 * j] + B_s[g * R + h + 2 * j];
-                        const float hi = v[2 * j + 1] + B_s[g * R + h + 2 * j + 1];
+                        const float lo = v[2 * j] + B_s[col + 2 * j];
+                        const float hi = v[2 * j + 1] + B_s[col + 2 * j + 1];
                         pk[j] = (uint32_t)from_f32<uint16_t>(lo) | ((uint32_t)from_f32<uint16_t>(hi) << 16);
                     }
-                    uint4 *dst = reinterpret_cast<uint4 *>(a.Y + n * a.M + (int64_t)row * R + h);
+                    uint4 *dst = reinterpret_cast<uint4 *>(a.Y + n * a.M + (int64_t)row * R + hr);
                     dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                     dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 } else {
-                    float4 *dst = reinterpret_cast<float4 *>(a.ws + ((int64_t)slot * a.N + n) * R + h);
+                    float4 *dst = reinterpret_cast<float4 *>(a.ws + ((int64_t)slot * a.N + n) * R + hr);
 #pragma unroll
                     for (int j = 0; j < 4; j++) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                 }
@@ -358,8 +384,8 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.n_items = n_items;
     a.G = G;
     a.n_tasks = (n_items + G - 1) / G;
-    a.rec = sc.d_xs_rec;
-    a.rec_off = sc.d_xs_rec_off;
+    a.trec = sc.tc.d_rec[gidx];
+    a.trec_off = sc.tc.d_rec_off[gidx];
     a.wpk = static_cast<const uint16_t *>(la.data);
     a.bias = la.bias;
     a.Y = static_cast<uint16_t *>(la.Y);
@@ -371,10 +397,10 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.C = sc.C;
     a.nchunks = (int)((sc.K + KC - 1) / KC);
     a.w_off = NS * kStageBytes;
-    a.rec_off_smem = a.w_off + (uint32_t)((sc.tc.task_wbytes[gidx] + 15) & ~size_t(15));
-    a.bias_off = a.rec_off_smem + (uint32_t)((sc.tc.task_ibytes[gidx] + 15) & ~size_t(15));
+    a.trec_smem = a.w_off + (uint32_t)((sc.tc.task_wbytes[gidx] + 15) & ~size_t(15));
+    a.bias_off = a.trec_smem + (uint32_t)((sc.tc.task_ibytes[gidx] + 15) & ~size_t(15));
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * R * 4 + 15) & ~size_t(15));
-    a.misc_off = a.bar_off + (2 * NS + 2) * 8;
+    a.misc_off = a.bar_off + (2 * NS + 3) * 8;
     a.tmem_cols = tmem_cols_for(G * R);
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
@@ -421,7 +447,7 @@ int tc_g_index(int G) {
 
 size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes) {
     return (size_t)NS * kStageBytes + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 2) * 8 + (4 + 6 * 32) * 4 + 1024;
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 3) * 8 + (4 + 6 * 32) * 4 + 1024;
 }
 
 size_t tc_task_budget(int R) {

@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <vector>
 
 #include "bsr.h"
 
@@ -16,10 +17,23 @@ constexpr int kTcTmemCols = 512;       // accumulator columns per SM
 constexpr int kTcTaskSizes = 6;
 constexpr int kTcG[kTcTaskSizes] = {1, 2, 4, 8, 16, 32};
 
+// Per task size G: the task records the kernel bulk-copies (see below), and
+// the largest block-value / record footprint of a task.
 struct TcPlan {
     size_t task_wbytes[kTcTaskSizes] = {0, 0, 0, 0, 0, 0};
     size_t task_ibytes[kTcTaskSizes] = {0, 0, 0, 0, 0, 0};
+    std::vector<int32_t> rec[kTcTaskSizes];       // all task records of this G
+    std::vector<int32_t> rec_off[kTcTaskSizes];   // per task: offset (ints, multiple of 4)
+    int32_t *d_rec[kTcTaskSizes] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+    int32_t *d_rec_off[kTcTaskSizes] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
 };
+
+// A task record (int32): [ per K chunk c = 0..nchunks: index of the chunk's
+// first entry, padded to 4 | one entry per MMA-block, chunk by chunk, padded
+// to 4 ]. Entry bits: [0,2) stage column offset / 32 bytes, [2,7) item in
+// the task, 7 first block of its item, [8,32) block index in the task's
+// block values.
+inline int64_t tc_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
 bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 int tc_g_index(int G);
