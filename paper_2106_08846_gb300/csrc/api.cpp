@@ -119,6 +119,7 @@ Schedule::~Schedule() {
     cudaFree(d_indptr);
     cudaFree(d_xs_rec);
     cudaFree(d_xs_rec_off);
+    cudaFree(d_xs_voff);
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);
         cudaFree(tc.d_rec_off[gi]);

@@ -69,8 +69,11 @@ struct Schedule {
     int32_t *d_group_begin = nullptr;
     std::vector<int32_t> xs_rec;        // xstage: per-item records (block offsets/columns, chunk starts)
     std::vector<int32_t> xs_rec_off;    // per item: record offset in ints (multiple of 4)
+    std::vector<int32_t> xs_voff;       // per item: offset of its packed block values, in 16-byte units
+    int64_t xs_values = 0;              // packed block values in floats (items padded to 16 bytes)
     int32_t *d_xs_rec = nullptr;
     int32_t *d_xs_rec_off = nullptr;
+    int32_t *d_xs_voff = nullptr;
     int32_t *d_indptr = nullptr;        // owned copies of the structure
     int32_t *d_indices = nullptr;
 
@@ -124,8 +127,8 @@ cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
 cudaError_t pack_tc_data(const void *data, int64_t nnzb, int R, int C, uint16_t *out, cudaStream_t s);
-cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, float *wpk,
-                             cudaStream_t s);
+cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *voff,
+                             int64_t n_items, int R, int C, float *wpk, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);
 int launches_per_call(const Schedule &sc);
 

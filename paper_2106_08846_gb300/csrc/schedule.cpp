@@ -101,8 +101,9 @@ void build_records(Schedule &sc, int chunk, F value) {
     }
 }
 
-// For each task size G, the largest block-value and record footprint over
-// the tasks formed by G consecutive items.
+// For each task size G, the largest block-value and record footprint (bytes,
+// each item's values padded to 16 bytes) over the tasks formed by G
+// consecutive items.
 void footprints(const Schedule &sc, size_t per_block, int chunk, const int *Gs, int nG, size_t *wbytes,
                 size_t *ibytes) {
     const int64_t nch = (sc.K + chunk - 1) / chunk;
@@ -113,10 +114,10 @@ void footprints(const Schedule &sc, size_t per_block, int chunk, const int *Gs, 
             size_t blocks = 0, rec = 0;
             for (size_t k = t; k < std::min(sc.items.size(), t + G); k++) {
                 const int64_t len = sc.items[k].p1 - sc.items[k].p0;
-                blocks += (size_t)len;
+                blocks += (size_t)xstage_pad4(len * (int64_t)per_block / 4) * 4;
                 rec += (size_t)xstage_record_ints(len, nch) * 4;
             }
-            wmax = std::max(wmax, blocks * per_block);
+            wmax = std::max(wmax, blocks);
             imax = std::max(imax, rec);
         }
         wbytes[gi] = wmax;
@@ -128,6 +129,14 @@ void plan_xstage(Schedule &sc) {
     build_records(sc, kXsChunk, [&](int64_t col) {
         return sc.C == 1 ? (int32_t)xstage_stage_offset(sc.dt, (int)(col % kXsChunk)) : (int32_t)col;
     });
+    // every item's block values start on a 16-byte boundary: one bulk copy each
+    sc.xs_voff.assign(sc.items.size(), 0);
+    int64_t off = 0;
+    for (size_t i = 0; i < sc.items.size(); i++) {
+        sc.xs_voff[i] = (int32_t)std::min<int64_t>(off / 4, INT32_MAX);
+        off += xstage_pad4((int64_t)(sc.items[i].p1 - sc.items[i].p0) * sc.R * sc.C * kXsWDup);
+    }
+    sc.xs_values = off;
     footprints(sc, (size_t)sc.R * sc.C * 4 * kXsWDup, kXsChunk, kXsG, kXsTaskSizes, sc.xs.task_wbytes,
                sc.xs.task_ibytes);
 }
@@ -220,8 +229,13 @@ bsr_status_t build_schedule(Schedule &sc) {
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
         make_items(sc, limit);
         plan_xstage(sc);
-    } else {
-        sc.variant = V_GENERIC;
+    }
+    if (sc.variant == V_XSTAGE && sc.xs_values / 4 > INT32_MAX) sc.variant = V_GENERIC;   // value offsets are int32
+    if (sc.variant == V_GENERIC) {
+        sc.threads = 256;
+        sc.xs_rec.clear();
+        sc.xs_rec_off.clear();
+        sc.xs_voff.clear();
         sc.tn = std::max(1, 256 / std::min(sc.R, 256));
         make_items(sc, split_limit(sc));
     }
@@ -229,7 +243,8 @@ bsr_status_t build_schedule(Schedule &sc) {
     if (upload(&sc.d_items, sc.items) != cudaSuccess || upload(&sc.d_splits, sc.splits) != cudaSuccess ||
         upload(&sc.d_group_begin, sc.group_begin) != cudaSuccess ||
         upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess ||
-        upload(&sc.d_xs_rec, sc.xs_rec) != cudaSuccess || upload(&sc.d_xs_rec_off, sc.xs_rec_off) != cudaSuccess) {
+        upload(&sc.d_xs_rec, sc.xs_rec) != cudaSuccess || upload(&sc.d_xs_rec_off, sc.xs_rec_off) != cudaSuccess ||
+        upload(&sc.d_xs_voff, sc.xs_voff) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
@@ -246,8 +261,7 @@ bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
     const Schedule &sc = *h.sched;
     if ((sc.variant != V_XSTAGE && sc.variant != V_TC) || sc.nnzb == 0) return BSR_OK;
-    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * sc.R * sc.C * 2
-                                            : (size_t)sc.nnzb * sc.R * sc.C * 4 * kXsWDup;
+    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * sc.R * sc.C * 2 : (size_t)sc.xs_values * 4;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
         h.data_packed = nullptr;
@@ -255,7 +269,8 @@ bsr_status_t pack_data(Handle &h) {
     }
     cudaError_t e = sc.variant == V_TC
                         ? pack_tc_data(h.data, sc.nnzb, sc.R, sc.C, (uint16_t *)h.data_packed, 0)
-                        : pack_xstage_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, (float *)h.data_packed, 0);
+                        : pack_xstage_data(h.data, sc.dt, sc.d_items, sc.d_xs_voff, (int64_t)sc.items.size(), sc.R,
+                                           sc.C, (float *)h.data_packed, 0);
     if (e != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_CUDA;

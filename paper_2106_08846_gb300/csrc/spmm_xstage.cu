@@ -54,6 +54,11 @@ constexpr int NS = kXsStages;
 constexpr int NCW = kXsConsumerWarps;
 constexpr int NTHREADS = (NCW + 1) * 32;
 constexpr int WD = kXsWDup;
+constexpr int kItab = 8;   // ints per item in the shared item table
+#ifndef XS_UNROLL
+#define XS_UNROLL 1
+#endif
+constexpr int kUnroll = XS_UNROLL;   // unrolling of the one-column block loop
 constexpr uint64_t kDrainNs = 200000000ull;   // bound for TMA loads already issued (they take microseconds)
 
 struct XsArgs {
@@ -61,7 +66,7 @@ struct XsArgs {
     int n_items, G, S, n_tasks;
     const int32_t *rec;      // per-item records (xstage_record_ints)
     const int32_t *rec_off;  // per item: record offset in ints
-    const float *wpk;        // [nnzb][C][R][WD]
+    const float *wpk;        // per item, 16-byte aligned: [block][C][R][WD]
     const float *bias;
     void *Y;
     float *ws;
@@ -69,7 +74,7 @@ struct XsArgs {
     int64_t N, K, M;
     int C, nchunks;
     uint32_t w_off, idx_off, bias_off, bar_off, misc_off;
-    int w_bulk;              // block values arrive by one bulk copy per item
+    const int32_t *voff;     // per item: offset of its packed values in 16-byte units
     uint64_t wait_ns;
     int stall_chunk;         // test hook: this chunk is never loaded (-1: none)
 };
@@ -138,10 +143,8 @@ struct Tile {
 #pragma unroll
         for (int k = 0; k < 4 * TR; k++) a[k] = 0ull;
     }
-    __device__ __forceinline__ void fma(const float (&x)[8], const float (&w)[TR]) {
-        f2_t wd[TR];
-#pragma unroll
-        for (int j = 0; j < TR; j++) wd[j] = pack2(w[j], w[j]);
+    // wd[j] = (w_j, w_j): the weight of output j, duplicated for both tokens
+    __device__ __forceinline__ void fma(const float (&x)[8], const f2_t (&wd)[TR]) {
 #pragma unroll
         for (int ip = 0; ip < 4; ip++) {
             const f2_t xp = pack2(x[2 * ip], x[2 * ip + 1]);
@@ -156,24 +159,37 @@ struct Tile {
     }
 };
 
-// the TR weights of one block column for this lane
+// The TR weights of one block column for this lane, each as a (w, w) pair.
+// With WD == 2 the packed values already hold every weight twice, so the
+// pairs come straight from shared loads.
 template <int TR>
-__device__ __forceinline__ void load_wd(const float *wr, float (&w)[TR]) {
-    if constexpr (TR % 4 == 0) {
+__device__ __forceinline__ void load_wd(const float *wr, f2_t (&wd)[TR]) {
+    if constexpr (WD == 2) {
+        if constexpr (TR == 1) {
+            wd[0] = *reinterpret_cast<const f2_t *>(wr);
+        } else {
+#pragma unroll
+            for (int j = 0; j < TR; j += 2) {
+                const ulonglong2 v = *reinterpret_cast<const ulonglong2 *>(wr + 2 * j);
+                wd[j] = v.x;
+                wd[j + 1] = v.y;
+            }
+        }
+    } else if constexpr (TR % 4 == 0) {
 #pragma unroll
         for (int j = 0; j < TR; j += 4) {
             const float4 v = *reinterpret_cast<const float4 *>(wr + j);
-            w[j] = v.x;
-            w[j + 1] = v.y;
-            w[j + 2] = v.z;
-            w[j + 3] = v.w;
+            wd[j] = pack2(v.x, v.x);
+            wd[j + 1] = pack2(v.y, v.y);
+            wd[j + 2] = pack2(v.z, v.z);
+            wd[j + 3] = pack2(v.w, v.w);
         }
     } else if constexpr (TR == 2) {
         const float2 v = *reinterpret_cast<const float2 *>(wr);
-        w[0] = v.x;
-        w[1] = v.y;
+        wd[0] = pack2(v.x, v.x);
+        wd[1] = pack2(v.y, v.y);
     } else {
-        w[0] = wr[0];
+        wd[0] = pack2(wr[0], wr[0]);
     }
 }
 
@@ -187,7 +203,7 @@ struct Shared {
     unsigned char *base;
     uint64_t *full, *empty, *wbar;
     int *misc;          // [0] abort flag
-    int *itab;          // per item: row p0 p1 slot rec_off len
+    int *itab;          // per item (kItab ints): row p0 p1 slot rec_off len voff16
     float *W;           // block values of the task's items
     int32_t *I;         // the task's item records
     float *B;           // [item][R] bias
@@ -198,8 +214,8 @@ __device__ __forceinline__ void item_offsets(const int *itab, int g, int per_blo
     woff = 0;
     roff = 0;
     for (int k = 0; k < g; k++) {
-        const int len = itab[6 * k + 5];
-        woff += len * per_block;
+        const int len = itab[kItab * k + 5];
+        woff += (int)xstage_pad4((int64_t)len * per_block);
         roff += (int)xstage_record_ints(len, nch);
     }
 }
@@ -214,17 +230,9 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     const int nch = a.nchunks;
     const int ctid = threadIdx.x;   // 0 .. NCW*32-1
 
-    // ---- bias (and block values when they cannot come by bulk copy); the
-    // records and block values arrive by the producer's bulk copies
+    // ---- bias; the records and block values arrive by the producer's bulk copies
     for (int g = 0; g < g_count; g++) {
-        if (!a.w_bulk) {
-            int woff, roff;
-            item_offsets(sh.itab, g, R * C * WD, nch, woff, roff);
-            const int p0 = sh.itab[6 * g + 1], len = sh.itab[6 * g + 5];
-            const float *src = a.wpk + (int64_t)p0 * R * C * WD;
-            for (int e = ctid; e < len * R * C * WD; e += NCW * 32) sh.W[woff + e] = __ldg(src + e);
-        }
-        const int64_t m0 = (int64_t)sh.itab[6 * g + 0] * R;
+        const int64_t m0 = (int64_t)sh.itab[kItab * g + 0] * R;
         for (int e = ctid; e < R; e += NCW * 32) sh.B[g * R + e] = a.bias ? __ldg(a.bias + m0 + e) : 0.f;
     }
     ptx::named_barrier(1, NCW * 32);
@@ -238,7 +246,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     int woff = 0, roff = 0;
     if (has_item) item_offsets(sh.itab, gi, R * C * WD, nch, woff, roff);
     const int32_t *idx = sh.I + roff;
-    const int32_t *cb = idx + (has_item ? xstage_pad4(sh.itab[6 * gi + 5]) : 0);
+    const int32_t *cb = idx + (has_item ? xstage_pad4(sh.itab[kItab * gi + 5]) : 0);
     const float *wbase = sh.W + woff + rg * TR * WD;
     const uint32_t tgx = (uint32_t)tg << 4;
     const unsigned char *lane_base = sh.base + tg * 128;
@@ -256,33 +264,16 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
             const int j0 = lo <= piece ? 0 : (lo - piece + S - 1) / S;
             const int j1 = hi <= piece ? 0 : (hi - piece + S - 1) / S;
             if constexpr (CT == 1) {
-                // one block ahead: the next block's operands are loaded while
-                // the current block's FMAs issue
-                int jj = j0 + ks;
-                if (jj < j1) {
-                    float xn[8], wn[TR];
-                    {
-                        const int lb = piece + S * jj;
-                        const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
+#pragma unroll kUnroll
+                for (int jj = j0 + ks; jj < j1; jj += NKS) {
+                    const int lb = piece + S * jj;
+                    const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
+                    float x[8];
+                    f2_t wd[TR];
 #pragma unroll
-                        for (int i = 0; i < 8; i++) xn[i] = ld_x(xp + i * 1024, T());
-                        load_wd<TR>(wbase + lb * R * WD, wn);
-                    }
-                    for (; jj < j1; jj += NKS) {
-                        float xc[8], wc[TR];
-#pragma unroll
-                        for (int i = 0; i < 8; i++) xc[i] = xn[i];
-#pragma unroll
-                        for (int j = 0; j < TR; j++) wc[j] = wn[j];
-                        if (jj + NKS < j1) {
-                            const int lb = piece + S * (jj + NKS);
-                            const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
-#pragma unroll
-                            for (int i = 0; i < 8; i++) xn[i] = ld_x(xp + i * 1024, T());
-                            load_wd<TR>(wbase + lb * R * WD, wn);
-                        }
-                        acc.fma(xc, wc);
-                    }
+                    for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
+                    load_wd<TR>(wbase + lb * R * WD, wd);
+                    acc.fma(x, wd);
                 }
             } else {
                 const int kbase = c * KC;
@@ -290,7 +281,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
                     const int lb = piece + S * jj;
                     const int kk = idx[lb] * C - kbase;
                     const float *wb = wbase + lb * C * R * WD;
-                    if ((C & 3) == 0) {
+                    if (TR < 8 && (C & 3) == 0) {   // four columns per load, where registers allow
                         for (int c4 = 0; c4 < C; c4 += 4) {
                             const unsigned char *xp = st + (St::off0(kk + c4) ^ tgx);
                             float4 xv[8];
@@ -299,7 +290,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
 #pragma unroll
                             for (int u = 0; u < 4; u++) {
                                 float x[8];
-                                float wd[TR];
+                                f2_t wd[TR];
 #pragma unroll
                                 for (int i = 0; i < 8; i++)
                                     x[i] = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
@@ -311,7 +302,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
                         for (int cc = 0; cc < C; cc++) {
                             const unsigned char *xp = st + (St::off0(kk + cc) ^ tgx);
                             float x[8];
-                            float wd[TR];
+                            f2_t wd[TR];
 #pragma unroll
                             for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
                             load_wd<TR>(wb + cc * R * WD, wd);
@@ -391,7 +382,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         ptx::named_barrier(1, NCW * 32);
     }
     if (!has_item || piece != 0 || ks != 0) return;
-    const int row = sh.itab[6 * gi + 0], slot = sh.itab[6 * gi + 3];
+    const int row = sh.itab[kItab * gi + 0], slot = sh.itab[kItab * gi + 3];
     const int64_t m = (int64_t)row * R + rg * TR;
     float b[TR];
 #pragma unroll
@@ -470,12 +461,13 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     if ((int)threadIdx.x < g_count) {   // one thread per item fills the item table
         const int g = threadIdx.x;
         const Item it = a.items[item_first + g];
-        sh.itab[6 * g + 0] = it.row;
-        sh.itab[6 * g + 1] = it.p0;
-        sh.itab[6 * g + 2] = it.p1;
-        sh.itab[6 * g + 3] = it.slot;
-        sh.itab[6 * g + 4] = __ldg(a.rec_off + item_first + g);
-        sh.itab[6 * g + 5] = it.p1 - it.p0;
+        sh.itab[kItab * g + 0] = it.row;
+        sh.itab[kItab * g + 1] = it.p0;
+        sh.itab[kItab * g + 2] = it.p1;
+        sh.itab[kItab * g + 3] = it.slot;
+        sh.itab[kItab * g + 4] = __ldg(a.rec_off + item_first + g);
+        sh.itab[kItab * g + 5] = it.p1 - it.p0;
+        sh.itab[kItab * g + 6] = __ldg(a.voff + item_first + g);
     }
     // every CTA's barriers exist before any multicast or remote arrive
     if (CL == 1) __syncthreads(); else ptx::cluster_sync();
@@ -488,20 +480,19 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
                 const int per_block = R * C * WD;
                 uint32_t total = 0;
                 for (int g = 0; g < g_count; g++) {
-                    const int len = sh.itab[6 * g + 5];
-                    total += (uint32_t)xstage_record_ints(len, nch) * 4;
-                    if (a.w_bulk) total += (uint32_t)len * per_block * 4;
+                    const int len = sh.itab[kItab * g + 5];
+                    total += (uint32_t)(xstage_record_ints(len, nch) + xstage_pad4((int64_t)len * per_block)) * 4;
                 }
                 ptx::mbar_arrive_expect_tx(sh.wbar, total);
                 int woff = 0, roff = 0;
                 for (int g = 0; g < g_count; g++) {
-                    const int len = sh.itab[6 * g + 5];
-                    const uint32_t wbytes = (uint32_t)len * per_block * 4;
-                    if (a.w_bulk && wbytes)
-                        ptx::bulk_load(sh.W + woff, a.wpk + (int64_t)sh.itab[6 * g + 1] * per_block, wbytes, sh.wbar);
+                    const int len = sh.itab[kItab * g + 5];
+                    const int wfl = (int)xstage_pad4((int64_t)len * per_block);
+                    if (wfl)
+                        ptx::bulk_load(sh.W + woff, a.wpk + (int64_t)sh.itab[kItab * g + 6] * 4, (uint32_t)wfl * 4, sh.wbar);
                     const int rints = (int)xstage_record_ints(len, nch);
-                    ptx::bulk_load(sh.I + roff, a.rec + sh.itab[6 * g + 4], (uint32_t)rints * 4, sh.wbar);
-                    woff += len * per_block;
+                    ptx::bulk_load(sh.I + roff, a.rec + sh.itab[kItab * g + 4], (uint32_t)rints * 4, sh.wbar);
+                    woff += wfl;
                     roff += rints;
                 }
             }
@@ -542,19 +533,24 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
 }
 
-// W^T per block, widened to fp32 (WD copies of each value):
-// wpk[((p*C + c)*R + r)*WD + d] = data[(p*R + r)*C + c].
+// Block values in the kernel's layout: item by item (each item starting on a
+// 16-byte boundary), per block W^T widened to fp32 with WD copies of each
+// value: wpk[4*voff[i] + ((b*C + c)*R + r)*WD + d] = data[((p0_i + b)*R + r)*C + c].
 template <typename T>
-__global__ void k_pack(const T *__restrict__ data, float *__restrict__ wpk, int64_t nnzb, int R, int C) {
-    const int64_t total = nnzb * R * C;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t p = e / ((int64_t)R * C);
-        const int rc = (int)(e - p * R * C);
-        const int c = rc / R, r = rc - c * R;
-        const float w = to_f32(data[(p * R + r) * C + c]);
+__global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ items, const int32_t *__restrict__ voff,
+                       int64_t n_items, float *__restrict__ wpk, int R, int C) {
+    for (int64_t i = blockIdx.x; i < n_items; i += gridDim.x) {
+        const Item it = items[i];
+        const int64_t total = (int64_t)(it.p1 - it.p0) * R * C;
+        float *dst = wpk + 4 * (int64_t)voff[i];
+        for (int64_t e = threadIdx.x; e < total; e += blockDim.x) {
+            const int64_t b = e / ((int64_t)R * C);
+            const int rc = (int)(e - b * R * C);
+            const int c = rc / R, r = rc - c * R;
+            const float w = to_f32(data[((it.p0 + b) * R + r) * C + c]);
 #pragma unroll
-        for (int d = 0; d < WD; d++) wpk[WD * e + d] = w;
+            for (int d = 0; d < WD; d++) dst[WD * e + d] = w;
+        }
     }
 }
 
@@ -657,9 +653,8 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.bias_off = a.idx_off + (uint32_t)((pl.task_ibytes[gidx] + 15) & ~size_t(15));
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * sc.R * 4 + 15) & ~size_t(15));
     a.misc_off = a.bar_off + (2 * NS + 1) * 8;
-    // one bulk copy per item needs every item's byte range 16-byte aligned
-    a.w_bulk = (sc.R * sc.C * WD * 4) % 16 == 0;
-    const uint32_t smem = a.misc_off + (4 + 6 * NCW) * 4 + 1024;   // + slack to align the base
+    a.voff = sc.d_xs_voff;
+    const uint32_t smem = a.misc_off + (4 + kItab * NCW) * 4 + 1024;   // + slack to align the base
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
     static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
@@ -740,7 +735,7 @@ size_t xstage_smem_bytes(bsr_dtype_t dt, int R, int64_t K, int G, size_t wbytes,
     const size_t nch = (size_t)((K + KC - 1) / KC);
     (void)nch;
     return region_bytes(dt, R) + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + (4 + 6 * NCW) * 4 + 1024;
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + (4 + kItab * NCW) * 4 + 1024;
 }
 
 size_t xstage_task_budget(bsr_dtype_t dt, int R, int64_t K) {
@@ -765,15 +760,14 @@ bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
     return r_ok && c_ok && K % align == 0 && K > 0;
 }
 
-cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, float *wpk,
-                             cudaStream_t s) {
-    const int64_t total = nnzb * R * C;
-    if (total == 0) return cudaSuccess;
-    const int grid = (int)std::min<int64_t>((total + 255) / 256, 1 << 20);
+cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *voff,
+                             int64_t n_items, int R, int C, float *wpk, cudaStream_t s) {
+    if (n_items == 0) return cudaSuccess;
+    const int grid = (int)std::min<int64_t>(n_items, 1 << 16);
     if (dt == BSR_F32)
-        k_pack<float><<<grid, 256, 0, s>>>((const float *)data, wpk, nnzb, R, C);
+        k_pack<float><<<grid, 256, 0, s>>>((const float *)data, items, voff, n_items, wpk, R, C);
     else
-        k_pack<uint16_t><<<grid, 256, 0, s>>>((const uint16_t *)data, wpk, nnzb, R, C);
+        k_pack<uint16_t><<<grid, 256, 0, s>>>((const uint16_t *)data, items, voff, n_items, wpk, R, C);
     return cudaGetLastError();
 }
 
