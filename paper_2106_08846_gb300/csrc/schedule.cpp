@@ -6,7 +6,8 @@
 // mean are split into pieces whose fp32 partial tiles are summed by a reduce
 // pass in a fixed order (so results do not depend on timing). Empty rows stay
 // as items so that their outputs receive the bias. Items are ordered longest
-// first, the classic LPT rule, so that the long ones start early.
+// first, the classic LPT rule, so that the long ones start early (except for
+// one-row blocks, which keep row order).
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
@@ -29,7 +30,8 @@ cudaError_t upload(T **dst, const std::vector<T> &v) {
     return cudaMemcpy(*dst, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice);
 }
 
-// Splits rows longer than `limit` blocks into ceil(len/limit) near-equal pieces.
+// Splits rows longer than `limit` blocks into ceil(len/limit) near-equal
+// pieces; orders the items longest first (LPT).
 void make_items(Schedule &sc, int64_t limit) {
     sc.items.clear();
     sc.splits.clear();
@@ -50,6 +52,10 @@ void make_items(Schedule &sc, int64_t limit) {
         }
         sc.splits.push_back(s);
     }
+    // One-row blocks keep row order: their tasks are many short rows, which
+    // averages out length differences, and consecutive rows let a task store
+    // whole row segments of Y.
+    if (sc.R == 1) return;
     std::stable_sort(sc.items.begin(), sc.items.end(),
                      [](const Item &a, const Item &b) { return a.p1 - a.p0 > b.p1 - b.p0; });
 }
@@ -281,9 +287,11 @@ bsr_status_t pack_data(Handle &h) {
 int launches_per_call(const Schedule &sc) { return 1 + (sc.splits.empty() ? 0 : 1); }
 
 // Task size for this call: the G that minimises a simple cost model,
-// waves * (fixed CTA cost + G items of work), among the G whose shared
-// memory fits. One CTA runs per SM; a CTA's fixed cost (pipeline fill,
-// staging, epilogue) is worth about kOverheadItems average items.
+// waves * (fixed CTA cost + the work of G items), among the G whose shared
+// memory fits. One CTA runs per SM. Work is counted in multiply-adds per
+// token (blocks x R x C); a CTA's fixed cost (pipeline fill, streaming the
+// X tile, staging, epilogue) is worth about kFixed of them, which is about
+// two 32x1 rows of a 768-wide weight at 80% block sparsity.
 int choose_tasks(const Schedule &sc, int64_t N) {
     static const int forced = [] {
         const char *v = getenv("BSR_XS_G");
@@ -291,14 +299,16 @@ int choose_tasks(const Schedule &sc, int64_t N) {
     }();
     auto fits = [&](int G) {
         const int gi = g_index(G);
-        return xstage_smem_bytes(sc.dt, sc.R, sc.K, G, sc.xs.task_wbytes[gi], sc.xs.task_ibytes[gi]) <=
-               (size_t)kXsMaxSmem;
+        return xstage_task_size_ok(sc.R, G) &&
+               xstage_smem_bytes(sc.dt, sc.R, sc.K, G, sc.xs.task_wbytes[gi], sc.xs.task_ibytes[gi]) <=
+                   (size_t)kXsMaxSmem;
     };
     for (int gi = 0; gi < kXsTaskSizes; gi++)
         if (forced == kXsG[gi] && fits(forced)) return forced;
-    const double kOverheadItems = 2.0;
+    const double kFixed = 10000.0;
     const int64_t tiles = (N + kXsTokens - 1) / kXsTokens;
     const int64_t items = (int64_t)sc.items.size();
+    const double item_work = items ? (double)sc.nnzb * sc.R * sc.C / (double)items : 0.0;
     int best = 1;
     double best_cost = -1.0;
     for (int gi = 0; gi < kXsTaskSizes; gi++) {
@@ -306,7 +316,7 @@ int choose_tasks(const Schedule &sc, int64_t N) {
         if (!fits(G)) continue;
         const int64_t ctas = tiles * ((items + G - 1) / G);
         const double waves = (double)((ctas + sc.sm_count - 1) / sc.sm_count);
-        const double cost = waves * (kOverheadItems + (double)std::min<int64_t>(G, items));
+        const double cost = waves * (kFixed + (double)std::min<int64_t>(G, items) * item_work);
         if (best_cost < 0 || cost < best_cost) {
             best_cost = cost;
             best = G;

@@ -1,9 +1,11 @@
 // SIMT BSR x dense kernel with X staged through a TMA ring ("xstage").
 //
 // Each CTA owns a tile of TN = 64 tokens and a task of G work items (block
-// rows or pieces of rows, Section 2.2's kept blocks), S = 12/G consumer warps
-// per item (12 consumer warps and one producer warp). The inner product over the kept blocks is FP32-FMA bound, so the
-// design goal is a high share of packed FMAs among the issued instructions:
+// rows or pieces of rows, Section 2.2's kept blocks): S = 12/G consumer
+// warps per item for G <= 12, or G/12 whole items per warp for one-row
+// blocks (12 consumer warps and one producer warp). The inner product over
+// the kept blocks is FP32-FMA bound, so the design goal is a high share of
+// packed FMAs among the issued instructions:
 //
 //  * The CL CTAs of a thread-block cluster share one token tile (different
 //    tasks). X[n0 : n0+64, k0 : k0+128] chunks stream through a 3-stage
@@ -13,15 +15,17 @@
 //    mbarrier counts the bytes of all slices; every consumer warp waits for
 //    every chunk in order, processes all of its blocks that fall in it, and
 //    releases the stage on the "empty" mbarrier of every CTA in the cluster.
-//  * Per item, the producer fetches by bulk copy the block values (repacked
-//    at create time to fp32 [p][c][r]) and a record built on the host: each
-//    block's X offset inside a stage (1-column blocks) or block column, and
-//    the first block of every chunk, so the per-chunk loop has no search or
-//    test. The consumers load the bias meanwhile.
+//  * Per task, the consumer threads copy in, with 16-byte cp.async (many
+//    in flight: one bulk copy per task streamed far slower), the block
+//    values (repacked at create time to fp32 [p][c][r], each item 16-byte
+//    aligned) and the items' records built on the host: each block's X
+//    offset inside a stage (1-column blocks) or block column, and the first
+//    block of every chunk, so the per-chunk loop has no search or test.
 //  * Lane = tg + 8 q: tg picks 8 tokens (tg, tg+8, ..., tg+56: conflict-free
 //    under the swizzle, which XORs the 16-byte column group with tg), q
 //    splits into NRG output groups of TR rows and NKS = 4/NRG lanes that take
-//    alternate blocks. A lane accumulates an 8 x TR tile with packed
+//    alternate blocks (or, for wide blocks, a quarter or half of each
+//    block's columns). A lane accumulates an 8 x TR tile with packed
 //    fma.rn.f32x2 over pairs of tokens: (x_t, x_t') * (w, w).
 //  * Epilogue: shuffle-reduce the NKS partials, then sum the S warps of an
 //    item by a fixed pairwise tree through shared memory; the item's first
@@ -54,7 +58,7 @@ constexpr int NS = kXsStages;
 constexpr int NCW = kXsConsumerWarps;
 constexpr int NTHREADS = (NCW + 1) * 32;
 constexpr int WD = kXsWDup;
-constexpr int kItab = 8;   // ints per item in the shared item table
+constexpr int kItab = 12;  // ints per item in the shared item table
 #ifndef XS_UNROLL
 #define XS_UNROLL 1
 #endif
@@ -201,55 +205,270 @@ __device__ __forceinline__ bool aborted(const int *flag) {
 
 struct Shared {
     unsigned char *base;
-    uint64_t *full, *empty, *wbar;
+    uint64_t *full, *empty;
     int *misc;          // [0] abort flag
-    int *itab;          // per item (kItab ints): row p0 p1 slot rec_off len voff16
+    int *itab;          // per item (kItab ints): row p0 p1 slot rec_off len voff16 woff roff
     float *W;           // block values of the task's items
     int32_t *I;         // the task's item records
     float *B;           // [item][R] bias
 };
 
-// Offsets of item g's block values (floats) and record (ints) in shared memory.
-__device__ __forceinline__ void item_offsets(const int *itab, int g, int per_block, int nch, int &woff, int &roff) {
-    woff = 0;
-    roff = 0;
-    for (int k = 0; k < g; k++) {
-        const int len = itab[kItab * k + 5];
-        woff += (int)xstage_pad4((int64_t)len * per_block);
-        roff += (int)xstage_record_ints(len, nch);
+// The blocks of one item that fall in X chunk c, for one lane: blocks
+// piece + S*jj inside the chunk's range, lanes ks taking alternate ones.
+template <typename T, int TR, int NRG, int CT>
+__device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *st, const int32_t *idx,
+                                           const int32_t *cb, const float *wbase, int c, int piece, int S, int ks,
+                                           uint32_t tgx, int C) {
+    using St = Stage<T>;
+    constexpr int NKS = 4 / NRG;
+    constexpr int R = TR * NRG;
+    const int lo = cb[c], hi = cb[c + 1];
+    int j0 = lo, j1 = hi;
+    if (S > 1) {
+        j0 = lo <= piece ? 0 : (lo - piece + S - 1) / S;
+        j1 = hi <= piece ? 0 : (hi - piece + S - 1) / S;
+    }
+    if constexpr (CT == 1) {
+#pragma unroll kUnroll
+        for (int jj = j0 + ks; jj < j1; jj += NKS) {
+            const int lb = piece + S * jj;
+            const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
+            float x[8];
+            f2_t wd[TR];
+#pragma unroll
+            for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
+            load_wd<TR>(wbase + lb * R * WD, wd);
+            acc.fma(x, wd);
+        }
+    } else {
+        // wide blocks (a multiple of 4 columns per lane group): the NKS lane
+        // groups split each block's columns, so no lanes idle when a chunk
+        // holds fewer blocks than groups; narrow blocks: groups take
+        // alternate blocks
+        const int kbase = c * KC;
+        const bool csplit = NKS > 1 && C % (4 * NKS) == 0;
+        const int cw = csplit ? C / NKS : C;
+        const int cc0 = csplit ? ks * cw : 0;
+        for (int jj = csplit ? j0 : j0 + ks; jj < j1; jj += csplit ? 1 : NKS) {
+            const int lb = piece + S * jj;
+            const int kk = idx[lb] * C - kbase;
+            const float *wb = wbase + lb * C * R * WD;
+            if (TR < 8 && (cw & 3) == 0) {   // four columns per load, where registers allow
+                for (int c4 = cc0; c4 < cc0 + cw; c4 += 4) {
+                    const unsigned char *xp = st + (St::off0(kk + c4) ^ tgx);
+                    float4 xv[8];
+#pragma unroll
+                    for (int i = 0; i < 8; i++) xv[i] = ld_x4(xp + i * 1024, T());
+#pragma unroll
+                    for (int u = 0; u < 4; u++) {
+                        float x[8];
+                        f2_t wd[TR];
+#pragma unroll
+                        for (int i = 0; i < 8; i++)
+                            x[i] = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
+                        load_wd<TR>(wb + (c4 + u) * R * WD, wd);
+                        acc.fma(x, wd);
+                    }
+                }
+            } else {
+                for (int cc = cc0; cc < cc0 + cw; cc++) {
+                    const unsigned char *xp = st + (St::off0(kk + cc) ^ tgx);
+                    float x[8];
+                    f2_t wd[TR];
+#pragma unroll
+                    for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
+                    load_wd<TR>(wb + cc * R * WD, wd);
+                    acc.fma(x, wd);
+                }
+            }
+        }
     }
 }
 
-template <typename T, int TR, int NRG, int CT>
+// The lane's 8 x TR tile with the NKS block-splitting lanes summed in.
+template <int TR, int NRG>
+__device__ __forceinline__ void reduce_tile(const Tile<TR> &acc, float (&v)[8][TR]) {
+    constexpr int NKS = 4 / NRG;
+#pragma unroll
+    for (int i = 0; i < 8; i++)
+#pragma unroll
+        for (int j = 0; j < TR; j++) {
+            float t = acc.get(i, j);
+            if constexpr (NKS >= 2) t += __shfl_xor_sync(0xffffffffu, t, 8 * NRG);
+            if constexpr (NKS >= 4) t += __shfl_xor_sync(0xffffffffu, t, 16 * NRG);
+            v[i][j] = t;
+        }
+}
+
+// Item gi's finished tile: + bias, converted, to Y; or, for a piece of a
+// split row, the fp32 partial to its workspace slot.
+template <typename T, int TR, int NRG>
+__device__ __forceinline__ void store_tile(const XsArgs &a, const Shared &sh, const float (&v)[8][TR], int gi,
+                                           int64_t n0, int rg, int tg) {
+    constexpr int R = TR * NRG;
+    const int row = sh.itab[kItab * gi + 0], slot = sh.itab[kItab * gi + 3];
+    const int64_t m = (int64_t)row * R + rg * TR;
+    float b[TR];
+#pragma unroll
+    for (int j = 0; j < TR; j++) b[j] = slot < 0 ? sh.B[gi * R + rg * TR + j] : 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+        const int64_t n = n0 + tg + 8 * i;
+        if (n >= a.N) continue;
+        if (slot < 0) {
+            T *dst = reinterpret_cast<T *>(a.Y) + n * a.M + m;
+            if constexpr (sizeof(T) == 4 && TR % 4 == 0) {
+#pragma unroll
+                for (int j = 0; j < TR; j += 4)
+                    *reinterpret_cast<float4 *>(dst + j) =
+                        make_float4(v[i][j] + b[j], v[i][j + 1] + b[j + 1], v[i][j + 2] + b[j + 2], v[i][j + 3] + b[j + 3]);
+            } else if constexpr (sizeof(T) == 2 && TR % 4 == 0) {
+#pragma unroll
+                for (int j = 0; j < TR; j += 4) {
+                    uint2 pk;
+                    pk.x = (uint32_t)from_f32<T>(v[i][j] + b[j]) | ((uint32_t)from_f32<T>(v[i][j + 1] + b[j + 1]) << 16);
+                    pk.y = (uint32_t)from_f32<T>(v[i][j + 2] + b[j + 2]) |
+                           ((uint32_t)from_f32<T>(v[i][j + 3] + b[j + 3]) << 16);
+                    *reinterpret_cast<uint2 *>(dst + j) = pk;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < TR; j++) dst[j] = from_f32<T>(v[i][j] + b[j]);
+            }
+        } else {
+            float *dst = a.ws + ((int64_t)slot * a.N + n) * R + rg * TR;
+#pragma unroll
+            for (int j = 0; j < TR; j++) dst[j] = v[i][j];
+        }
+    }
+}
+
+// Consumer warps. RW == 1: S = 12/G warps share each item (block-strided)
+// and a pairwise tree sums them. RW > 1 (G = 12 RW): each warp owns RW
+// whole items, with one register tile each, and needs no tree.
+template <typename T, int TR, int NRG, int CT, int RW>
 __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int64_t n0, int item_first,
                                          int g_count, uint32_t CL, int warp, int lane) {
     using St = Stage<T>;
-    constexpr int NKS = 4 / NRG;
     constexpr int R = TR * NRG;
     const int C = CT ? CT : a.C;
     const int nch = a.nchunks;
     const int ctid = threadIdx.x;   // 0 .. NCW*32-1
 
-    // ---- bias; the records and block values arrive by the producer's bulk copies
-    for (int g = 0; g < g_count; g++) {
-        const int64_t m0 = (int64_t)sh.itab[kItab * g + 0] * R;
-        for (int e = ctid; e < R; e += NCW * 32) sh.B[g * R + e] = a.bias ? __ldg(a.bias + m0 + e) : 0.f;
+    // ---- each item's shared-memory offsets, then the task's block values
+    // and records (consecutive in memory: the task's items are consecutive)
+    // by 16-byte asynchronous copies from all consumer threads, and the bias
+    if (ctid < g_count) {
+        int woff = 0, roff = 0;
+        for (int k = 0; k <= ctid; k++) {
+            const int len = sh.itab[kItab * k + 5];
+            if (k == ctid) {
+                sh.itab[kItab * k + 7] = woff;
+                sh.itab[kItab * k + 8] = roff;
+            }
+            woff += (int)xstage_pad4((int64_t)len * R * C * WD);
+            roff += (int)xstage_record_ints(len, nch);
+        }
+        if (ctid == g_count - 1) {
+            sh.misc[1] = woff;   // floats
+            sh.misc[2] = roff;   // ints
+        }
+        // does the task cover consecutive whole rows? (then the epilogue
+        // stores whole row segments of Y)
+        if (sh.itab[kItab * ctid + 0] != sh.itab[0] + ctid || sh.itab[kItab * ctid + 3] >= 0) sh.misc[3] = 0;
     }
     ptx::named_barrier(1, NCW * 32);
-    bool ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(sh.wbar, 0, a.wait_ns));
+    if (g_count > 0) {
+        const int wq = sh.misc[1] / 4, rq = sh.misc[2] / 4;   // 16-byte pieces
+        const float4 *ws = reinterpret_cast<const float4 *>(a.wpk + (int64_t)sh.itab[6] * 4);
+        const int4 *rs = reinterpret_cast<const int4 *>(a.rec + sh.itab[4]);
+        for (int e = ctid; e < wq; e += NCW * 32) ptx::cp_async16(reinterpret_cast<float4 *>(sh.W) + e, ws + e);
+        for (int e = ctid; e < rq; e += NCW * 32) ptx::cp_async16(reinterpret_cast<int4 *>(sh.I) + e, rs + e);
+    }
+    for (int e = ctid; e < g_count * R; e += NCW * 32) {   // one bias value per thread: loads in parallel
+        const int g = e / R, r = e - g * R;
+        sh.B[e] = a.bias ? __ldg(a.bias + (int64_t)sh.itab[kItab * g + 0] * R + r) : 0.f;
+    }
+    ptx::cp_async_wait_all();
+    ptx::named_barrier(1, NCW * 32);
+    bool ok = true;
 
     const int q = lane >> 3, tg = lane & 7;
     const int rg = q % NRG, ks = q / NRG;
+    const uint32_t tgx = (uint32_t)tg << 4;
+    const unsigned char *lane_base = sh.base + tg * 128;
+
+    if constexpr (RW > 1) {
+        Tile<TR> acc[RW];
+#pragma unroll
+        for (int r = 0; r < RW; r++) acc[r].zero();
+        for (int c = 0; c < nch && ok; c++) {
+            const bool got = ptx::mbar_wait_bounded(&sh.full[c % NS], (c / NS) & 1, a.wait_ns) && !aborted(sh.misc);
+            ok = __all_sync(0xffffffffu, got);
+            if (!ok) break;
+            const unsigned char *st = lane_base + (c % NS) * St::kBytes;
+#pragma unroll
+            for (int r = 0; r < RW; r++) {
+                const int gi = warp * RW + r;
+                if (gi < g_count) {
+                    const int32_t *idx = sh.I + sh.itab[kItab * gi + 8];
+                    const int32_t *cb = idx + xstage_pad4(sh.itab[kItab * gi + 5]);
+                    const float *wbase = sh.W + sh.itab[kItab * gi + 7] + rg * TR * WD;
+                    item_chunk<T, TR, NRG, CT>(acc[r], st, idx, cb, wbase, c, 0, 1, ks, tgx, C);
+                }
+            }
+            __syncwarp();
+            if (CL == 1) {
+                if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
+            } else if (lane < (int)CL) {
+                ptx::mbar_arrive_cluster(ptx::mapa(ptx::smem_addr(&sh.empty[c % NS]), lane));
+            }
+        }
+        if (!ok && lane == 0) {
+            set_status(a.status, DEV_TIMEOUT);
+            atomicExch(&sh.misc[0], 1);
+        }
+        if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
+        if (R == 1 && sh.misc[3]) {
+            // consecutive rows row0 .. row0+G-1: transpose the tiles through
+            // shared memory (the ring is free) and store Y row segments
+            const int PG = g_count + 1;
+            float *P = reinterpret_cast<float *>(sh.base);
+#pragma unroll
+            for (int r = 0; r < RW; r++) {
+                const int gi = warp * RW + r;
+                float v[8][TR];
+                reduce_tile<TR, NRG>(acc[r], v);
+                if (gi < g_count && ks == 0)
+#pragma unroll
+                    for (int i = 0; i < 8; i++) P[(tg + 8 * i) * PG + gi] = v[i][0];
+            }
+            ptx::named_barrier(1, NCW * 32);
+            const int64_t row0 = sh.itab[0];
+            for (int e = ctid; e < TN * g_count; e += NCW * 32) {
+                const int t = e / g_count, j = e - t * g_count;
+                const int64_t n = n0 + t;
+                if (n < a.N)
+                    reinterpret_cast<T *>(a.Y)[n * a.M + row0 + j] = from_f32<T>(P[t * PG + j] + sh.B[j]);
+            }
+            return;
+        }
+#pragma unroll
+        for (int r = 0; r < RW; r++) {
+            const int gi = warp * RW + r;
+            float v[8][TR];
+            reduce_tile<TR, NRG>(acc[r], v);
+            if (gi < g_count && ks == 0) store_tile<T, TR, NRG>(a, sh, v, gi, n0, rg, tg);
+        }
+        return;
+    }
+
     const int S = a.S;
     const int gi = warp / S, piece = warp % S;
     const bool has_item = gi < g_count;
-    int woff = 0, roff = 0;
-    if (has_item) item_offsets(sh.itab, gi, R * C * WD, nch, woff, roff);
-    const int32_t *idx = sh.I + roff;
+    const int32_t *idx = sh.I + (has_item ? sh.itab[kItab * gi + 8] : 0);
     const int32_t *cb = idx + (has_item ? xstage_pad4(sh.itab[kItab * gi + 5]) : 0);
-    const float *wbase = sh.W + woff + rg * TR * WD;
-    const uint32_t tgx = (uint32_t)tg << 4;
-    const unsigned char *lane_base = sh.base + tg * 128;
+    const float *wbase = sh.W + (has_item ? sh.itab[kItab * gi + 7] : 0) + rg * TR * WD;
 
     Tile<TR> acc;
     acc.zero();
@@ -257,61 +476,8 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         const bool got = ptx::mbar_wait_bounded(&sh.full[c % NS], (c / NS) & 1, a.wait_ns) && !aborted(sh.misc);
         ok = __all_sync(0xffffffffu, got);
         if (!ok) break;
-        if (has_item) {
-            const unsigned char *st = lane_base + (c % NS) * St::kBytes;
-            const int lo = cb[c], hi = cb[c + 1];
-            // this warp's blocks piece + S*jj inside [lo, hi); lanes ks take alternate ones
-            const int j0 = lo <= piece ? 0 : (lo - piece + S - 1) / S;
-            const int j1 = hi <= piece ? 0 : (hi - piece + S - 1) / S;
-            if constexpr (CT == 1) {
-#pragma unroll kUnroll
-                for (int jj = j0 + ks; jj < j1; jj += NKS) {
-                    const int lb = piece + S * jj;
-                    const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
-                    float x[8];
-                    f2_t wd[TR];
-#pragma unroll
-                    for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
-                    load_wd<TR>(wbase + lb * R * WD, wd);
-                    acc.fma(x, wd);
-                }
-            } else {
-                const int kbase = c * KC;
-                for (int jj = j0 + ks; jj < j1; jj += NKS) {
-                    const int lb = piece + S * jj;
-                    const int kk = idx[lb] * C - kbase;
-                    const float *wb = wbase + lb * C * R * WD;
-                    if (TR < 8 && (C & 3) == 0) {   // four columns per load, where registers allow
-                        for (int c4 = 0; c4 < C; c4 += 4) {
-                            const unsigned char *xp = st + (St::off0(kk + c4) ^ tgx);
-                            float4 xv[8];
-#pragma unroll
-                            for (int i = 0; i < 8; i++) xv[i] = ld_x4(xp + i * 1024, T());
-#pragma unroll
-                            for (int u = 0; u < 4; u++) {
-                                float x[8];
-                                f2_t wd[TR];
-#pragma unroll
-                                for (int i = 0; i < 8; i++)
-                                    x[i] = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
-                                load_wd<TR>(wb + (c4 + u) * R * WD, wd);
-                                acc.fma(x, wd);
-                            }
-                        }
-                    } else {
-                        for (int cc = 0; cc < C; cc++) {
-                            const unsigned char *xp = st + (St::off0(kk + cc) ^ tgx);
-                            float x[8];
-                            f2_t wd[TR];
-#pragma unroll
-                            for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
-                            load_wd<TR>(wb + cc * R * WD, wd);
-                            acc.fma(x, wd);
-                        }
-                    }
-                }
-            }
-        }
+        if (has_item)
+            item_chunk<T, TR, NRG, CT>(acc, lane_base + (c % NS) * St::kBytes, idx, cb, wbase, c, piece, S, ks, tgx, C);
         __syncwarp();
         if (CL == 1) {
             if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
@@ -326,15 +492,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
 
     // ---- epilogue
     float v[8][TR];
-#pragma unroll
-    for (int i = 0; i < 8; i++)
-#pragma unroll
-        for (int j = 0; j < TR; j++) {
-            float t = acc.get(i, j);
-            if constexpr (NKS >= 2) t += __shfl_xor_sync(0xffffffffu, t, 8 * NRG);
-            if constexpr (NKS >= 4) t += __shfl_xor_sync(0xffffffffu, t, 16 * NRG);
-            v[i][j] = t;
-        }
+    reduce_tile<TR, NRG>(acc, v);
     // every consumer is done with the ring and the block values; the abort
     // verdict is the same for all of them (barrier reduction)
     if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
@@ -382,44 +540,10 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         ptx::named_barrier(1, NCW * 32);
     }
     if (!has_item || piece != 0 || ks != 0) return;
-    const int row = sh.itab[kItab * gi + 0], slot = sh.itab[kItab * gi + 3];
-    const int64_t m = (int64_t)row * R + rg * TR;
-    float b[TR];
-#pragma unroll
-    for (int j = 0; j < TR; j++) b[j] = slot < 0 ? sh.B[gi * R + rg * TR + j] : 0.f;
-#pragma unroll
-    for (int i = 0; i < 8; i++) {
-        const int64_t n = n0 + tg + 8 * i;
-        if (n >= a.N) continue;
-        if (slot < 0) {
-            T *dst = reinterpret_cast<T *>(a.Y) + n * a.M + m;
-            if constexpr (sizeof(T) == 4 && TR % 4 == 0) {
-#pragma unroll
-                for (int j = 0; j < TR; j += 4)
-                    *reinterpret_cast<float4 *>(dst + j) =
-                        make_float4(v[i][j] + b[j], v[i][j + 1] + b[j + 1], v[i][j + 2] + b[j + 2], v[i][j + 3] + b[j + 3]);
-            } else if constexpr (sizeof(T) == 2 && TR % 4 == 0) {
-#pragma unroll
-                for (int j = 0; j < TR; j += 4) {
-                    uint2 pk;
-                    pk.x = (uint32_t)from_f32<T>(v[i][j] + b[j]) | ((uint32_t)from_f32<T>(v[i][j + 1] + b[j + 1]) << 16);
-                    pk.y = (uint32_t)from_f32<T>(v[i][j + 2] + b[j + 2]) |
-                           ((uint32_t)from_f32<T>(v[i][j + 3] + b[j + 3]) << 16);
-                    *reinterpret_cast<uint2 *>(dst + j) = pk;
-                }
-            } else {
-#pragma unroll
-                for (int j = 0; j < TR; j++) dst[j] = from_f32<T>(v[i][j] + b[j]);
-            }
-        } else {
-            float *dst = a.ws + ((int64_t)slot * a.N + n) * R + rg * TR;
-#pragma unroll
-            for (int j = 0; j < TR; j++) dst[j] = v[i][j];
-        }
-    }
+    store_tile<T, TR, NRG>(a, sh, v, gi, n0, rg, tg);
 }
 
-template <typename T, int TR, int NRG, int CT>
+template <typename T, int TR, int NRG, int CT, int RW>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     using St = Stage<T>;
@@ -429,7 +553,6 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     sh.base = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     sh.full = reinterpret_cast<uint64_t *>(sh.base + a.bar_off);
     sh.empty = sh.full + NS;
-    sh.wbar = sh.empty + NS;
     sh.misc = reinterpret_cast<int *>(sh.base + a.misc_off);
     sh.itab = sh.misc + 4;
     sh.W = reinterpret_cast<float *>(sh.base + a.w_off);
@@ -454,8 +577,8 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
             ptx::mbar_init(&sh.full[s], 1);
             ptx::mbar_init(&sh.empty[s], NCW * CL);
         }
-        ptx::mbar_init(sh.wbar, 1);
         sh.misc[0] = 0;
+        sh.misc[3] = 1;
         ptx::fence_barrier_init();
     }
     if ((int)threadIdx.x < g_count) {   // one thread per item fills the item table
@@ -476,26 +599,6 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
         // ---------------- producer: block values by bulk copy, then X chunks
         if (lane == 0) {
             ptx::prefetch_tensormap(&xmap);
-            {
-                const int per_block = R * C * WD;
-                uint32_t total = 0;
-                for (int g = 0; g < g_count; g++) {
-                    const int len = sh.itab[kItab * g + 5];
-                    total += (uint32_t)(xstage_record_ints(len, nch) + xstage_pad4((int64_t)len * per_block)) * 4;
-                }
-                ptx::mbar_arrive_expect_tx(sh.wbar, total);
-                int woff = 0, roff = 0;
-                for (int g = 0; g < g_count; g++) {
-                    const int len = sh.itab[kItab * g + 5];
-                    const int wfl = (int)xstage_pad4((int64_t)len * per_block);
-                    if (wfl)
-                        ptx::bulk_load(sh.W + woff, a.wpk + (int64_t)sh.itab[kItab * g + 6] * 4, (uint32_t)wfl * 4, sh.wbar);
-                    const int rints = (int)xstage_record_ints(len, nch);
-                    ptx::bulk_load(sh.I + roff, a.rec + sh.itab[kItab * g + 4], (uint32_t)rints * 4, sh.wbar);
-                    woff += wfl;
-                    roff += rints;
-                }
-            }
             const int rows = TN / (int)CL;                       // this CTA's slice of every chunk
             const uint16_t mask = (uint16_t)((1u << CL) - 1u);
             int c = 0;
@@ -524,11 +627,10 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
             // them so that no TMA write outlives the CTA
             for (int d = max(0, c - NS); d < c; d++)
                 if (d != a.stall_chunk) ptx::mbar_wait_bounded(&sh.full[d % NS], (d / NS) & 1, kDrainNs);
-            ptx::mbar_wait_bounded(sh.wbar, 0, kDrainNs);
         }
         __syncwarp();
     } else {
-        consumer<T, TR, NRG, CT>(a, sh, n0, item_first, g_count, CL, warp, lane);
+        consumer<T, TR, NRG, CT, RW>(a, sh, n0, item_first, g_count, CL, warp, lane);
     }
     if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
 }
@@ -620,7 +722,7 @@ int choose_cluster(int n_tasks) {
     return 1;
 }
 
-template <typename T, int TR, int NRG, int CT>
+template <typename T, int TR, int NRG, int CT, int RW>
 cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     const Schedule &sc = *la.sc;
     const size_t es = sizeof(T);
@@ -634,7 +736,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.items = sc.d_items;
     a.n_items = n_items;
     a.G = G;
-    a.S = NCW / G;
+    a.S = G <= NCW ? NCW / G : 1;
     a.n_tasks = (n_items + G - 1) / G;
     a.rec = sc.d_xs_rec;
     a.rec_off = sc.d_xs_rec_off;
@@ -654,7 +756,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * sc.R * 4 + 15) & ~size_t(15));
     a.misc_off = a.bar_off + (2 * NS + 1) * 8;
     a.voff = sc.d_xs_voff;
-    const uint32_t smem = a.misc_off + (4 + kItab * NCW) * 4 + 1024;   // + slack to align the base
+    const uint32_t smem = a.misc_off + (4 + kItab * G) * 4 + 1024;   // + slack to align the base
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
     static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
@@ -662,7 +764,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     cudaGetDevice(&dev);
     const uint64_t bit = 1ull << (dev & 63);
     if (!(attr_set.load() & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG, CT>,
+        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG, CT, RW>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kXsMaxSmem);
         if (e != cudaSuccess) return e;
         attr_set.fetch_or(bit);
@@ -672,7 +774,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
 
     cudaError_t err = cudaErrorInvalidConfiguration;
     for (int CL = choose_cluster(a.n_tasks); CL >= 1; CL >>= 1) {
-        if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT>), CL, smem, dev))
+        if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT, RW>), CL, smem, dev))
             continue;
         const int64_t n_groups = (a.n_tasks + CL - 1) / CL;
         const int64_t grid = n_tiles * n_groups * CL;   // cluster-major, tile-fastest
@@ -688,7 +790,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
         if (CL == 1) {
-            k_xstage<T, TR, NRG, CT><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
+            k_xstage<T, TR, NRG, CT, RW><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
             err = cudaGetLastError();
             break;
         }
@@ -704,16 +806,29 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
         attr[0].val.clusterDim.z = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        err = cudaLaunchKernelEx(&cfg, k_xstage<T, TR, NRG, CT>, map, a);
+        err = cudaLaunchKernelEx(&cfg, k_xstage<T, TR, NRG, CT, RW>, map, a);
         break;
     }
     return err;
 }
 
+// Items per consumer warp: G = 12 RW with RW > 1 only for one-row blocks.
+template <typename T, int TR, int NRG, int CT>
+cudaError_t launch_w(const LaunchArgs &la, const XsPlan &pl, int G) {
+    if constexpr (TR == 1 && NRG == 1) {
+        switch (G / NCW) {
+            case 2: return launch_t<T, TR, NRG, CT, 2>(la, pl, G);
+            case 4: return launch_t<T, TR, NRG, CT, 4>(la, pl, G);
+        }
+    }
+    if (G > NCW) return cudaErrorInvalidConfiguration;
+    return launch_t<T, TR, NRG, CT, 1>(la, pl, G);
+}
+
 template <typename T, int TR, int NRG>
 cudaError_t launch_c(const LaunchArgs &la, const XsPlan &pl, int G) {
-    if (la.sc->C == 1) return launch_t<T, TR, NRG, 1>(la, pl, G);
-    return launch_t<T, TR, NRG, 0>(la, pl, G);
+    if (la.sc->C == 1) return launch_w<T, TR, NRG, 1>(la, pl, G);
+    return launch_w<T, TR, NRG, 0>(la, pl, G);
 }
 
 template <typename T>
@@ -735,7 +850,7 @@ size_t xstage_smem_bytes(bsr_dtype_t dt, int R, int64_t K, int G, size_t wbytes,
     const size_t nch = (size_t)((K + KC - 1) / KC);
     (void)nch;
     return region_bytes(dt, R) + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + (4 + kItab * NCW) * 4 + 1024;
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + (4 + kItab * (size_t)G) * 4 + 1024;
 }
 
 size_t xstage_task_budget(bsr_dtype_t dt, int R, int64_t K) {
@@ -752,6 +867,8 @@ int g_index(int G) {
         if (kXsG[i] == G) return i;
     return 0;
 }
+
+bool xstage_task_size_ok(int R, int G) { return G <= kXsConsumerWarps || R == 1; }
 
 bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
     const bool r_ok = R == 1 || R == 2 || R == 4 || R == 8 || R == 16 || R == 32;

@@ -15,15 +15,17 @@ constexpr int kXsConsumerWarps = 12;   // + 1 producer warp: 16 warps of registe
 constexpr int kXsMaxSmem = 232448;     // 227 KB, the per-CTA opt-in limit
 constexpr int kXsWDup = 1;             // copies of each packed block value
 
-// Task sizes G (items per CTA); each divides the consumer warps.
-constexpr int kXsTaskSizes = 6;
-constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12};
+// Task sizes G (items per CTA): up to 12, each divides the consumer warps
+// (12/G warps per item); above 12, each warp owns G/12 items (one-row
+// blocks only, whose register tiles are small).
+constexpr int kXsTaskSizes = 8;
+constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12, 24, 48};
 
 // Per task size (index into kXsG): the largest shared-memory footprint of
 // block values / indices over all tasks of G consecutive items.
 struct XsPlan {
-    size_t task_wbytes[kXsTaskSizes] = {0, 0, 0, 0, 0, 0};
-    size_t task_ibytes[kXsTaskSizes] = {0, 0, 0, 0, 0, 0};   // item records (see xstage_record_ints)
+    size_t task_wbytes[kXsTaskSizes] = {};
+    size_t task_ibytes[kXsTaskSizes] = {};   // item records (see xstage_record_ints)
 };
 
 // Per item, the kernel fetches one "record" of int32 by bulk copy:
@@ -43,6 +45,7 @@ XS_HD inline int64_t xstage_record_ints(int64_t len, int64_t nchunks) {
 uint32_t xstage_stage_offset(bsr_dtype_t dt, int kk);
 
 int g_index(int G);
+bool xstage_task_size_ok(int R, int G);   // G > 12 needs one-row blocks
 bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 
 // Dynamic shared memory of one CTA: ring (reused for the epilogue's partial
