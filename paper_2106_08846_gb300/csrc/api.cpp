@@ -117,9 +117,8 @@ Schedule::~Schedule() {
     cudaFree(d_splits);
     cudaFree(d_group_begin);
     cudaFree(d_indptr);
-    cudaFree(d_xs_rec);
-    cudaFree(d_xs_rec_off);
-    cudaFree(d_xs_voff);
+    cudaFree(d_xs_perm);
+    cudaFree(d_xs_vdst);
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);
         cudaFree(tc.d_rec_off[gi]);

@@ -69,11 +69,13 @@ struct Schedule {
     int32_t *d_group_begin = nullptr;
     std::vector<int32_t> xs_rec;        // xstage: per-item records (block offsets/columns, chunk starts)
     std::vector<int32_t> xs_rec_off;    // per item: record offset in ints (multiple of 4)
-    std::vector<int32_t> xs_voff;       // per item: offset of its packed block values, in 16-byte units
-    int64_t xs_values = 0;              // packed block values in floats (items padded to 16 bytes)
-    int32_t *d_xs_rec = nullptr;
-    int32_t *d_xs_rec_off = nullptr;
-    int32_t *d_xs_voff = nullptr;
+    std::vector<int32_t> xs_perm;       // per packed block position: the stored block it holds
+    std::vector<int32_t> xs_blob;       // task blobs of every task size, block values left zero
+    int64_t xs_blob_off[kXsTaskSizes] = {};      // byte offset of task size gi's blobs (-1: not usable)
+    int64_t xs_blob_stride[kXsTaskSizes] = {};   // bytes per task
+    std::vector<int64_t> xs_vdst;       // [gi][item]: float offset of the item's values in the blobs (-1: none)
+    int32_t *d_xs_perm = nullptr;
+    int64_t *d_xs_vdst = nullptr;
     int32_t *d_indptr = nullptr;        // owned copies of the structure
     int32_t *d_indices = nullptr;
 
@@ -127,8 +129,8 @@ cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
 cudaError_t pack_tc_data(const void *data, int64_t nnzb, int R, int C, uint16_t *out, cudaStream_t s);
-cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *voff,
-                             int64_t n_items, int R, int C, float *wpk, cudaStream_t s);
+cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
+                             const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);
 int launches_per_call(const Schedule &sc);
 

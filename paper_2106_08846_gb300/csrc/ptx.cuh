@@ -85,6 +85,12 @@ __device__ __forceinline__ void cp_async16(void *dst, const void *src) {
                  "l"(reinterpret_cast<uint64_t>(src))
                  : "memory");
 }
+// 4-byte asynchronous copy global -> shared (4-byte aligned addresses).
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst)),
+                 "l"(reinterpret_cast<uint64_t>(src))
+                 : "memory");
+}
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {

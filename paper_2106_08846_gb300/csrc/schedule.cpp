@@ -80,6 +80,47 @@ int64_t split_limit(const Schedule &sc) {
     return sc.max_row > limit ? limit : 0;
 }
 
+// One-column blocks: the lanes of a warp read the X columns of NKS (up to 4)
+// blocks at once; under the 128-byte swizzle two columns conflict in shared
+// memory when they share a residue (column mod 4 for fp32, (column / 2) mod 4
+// for bf16). Reorder the blocks [lo, hi) of one item's chunk so that every
+// aligned group of four has distinct residues where the counts allow:
+// repeatedly take one block from each of the fullest residue classes.
+void quad_order(Schedule &sc, int32_t p0, int32_t lo, int32_t hi) {
+    std::vector<int32_t> cls[4];
+    for (int32_t k = lo; k < hi; k++) {
+        const int32_t p = sc.xs_perm[(size_t)p0 + k];
+        const int64_t col = sc.indices[p];
+        const int r = (int)(sc.dt == BSR_F32 ? (col & 3) : ((col >> 1) & 3));
+        cls[r].push_back(p);
+    }
+    size_t at[4] = {0, 0, 0, 0};
+    int32_t k = lo;
+    while (k < hi) {
+        int order[4] = {0, 1, 2, 3};
+        std::sort(order, order + 4, [&](int a, int b) {
+            const size_t ra = cls[a].size() - at[a], rb = cls[b].size() - at[b];
+            return ra != rb ? ra > rb : a < b;
+        });
+        int taken = 0;
+        for (int t = 0; t < 4 && k < hi; t++) {
+            const int r = order[t];
+            if (at[r] < cls[r].size()) {
+                sc.xs_perm[(size_t)p0 + k++] = cls[r][at[r]++];
+                taken++;
+            }
+        }
+        // fewer than four classes left: fill the group from the fullest ones
+        for (int t = 0; taken < 4 && k < hi; t = (t + 1) % 4) {
+            const int r = order[t];
+            if (at[r] < cls[r].size()) {
+                sc.xs_perm[(size_t)p0 + k++] = cls[r][at[r]++];
+                taken++;
+            }
+        }
+    }
+}
+
 // For each task size G, the largest block-value and index footprint over
 // the tasks formed by G consecutive items of the (LPT-ordered) item list.
 // Per-item records fetched by the kernels: one int per block (`value` of its
@@ -90,13 +131,13 @@ void build_records(Schedule &sc, int chunk, F value) {
     const int64_t nch = (sc.K + chunk - 1) / chunk;
     sc.xs_rec.clear();
     sc.xs_rec_off.assign(sc.items.size(), 0);
+    sc.xs_perm.assign((size_t)sc.nnzb, 0);
     for (size_t i = 0; i < sc.items.size(); i++) {
         const Item &it = sc.items[i];
         const int32_t len = it.p1 - it.p0;
         sc.xs_rec_off[i] = (int32_t)sc.xs_rec.size();
         const size_t base = sc.xs_rec.size();
         sc.xs_rec.resize(base + (size_t)xstage_record_ints(len, nch), 0);
-        for (int32_t b = 0; b < len; b++) sc.xs_rec[base + b] = value((int64_t)sc.indices[it.p0 + b]);
         int32_t b = 0;
         const size_t cbase = base + (size_t)xstage_pad4(len);
         for (int64_t c = 0; c <= nch; c++) {
@@ -104,6 +145,13 @@ void build_records(Schedule &sc, int chunk, F value) {
             while (b < len && sc.indices[it.p0 + b] < first_col) b++;
             sc.xs_rec[cbase + c] = b;
         }
+        // block order inside each chunk (perm: position -> stored block)
+        for (int32_t k = 0; k < len; k++) sc.xs_perm[(size_t)it.p0 + k] = it.p0 + k;
+        if (sc.C == 1)
+            for (int64_t c = 0; c < nch; c++)
+                quad_order(sc, it.p0, sc.xs_rec[cbase + c], sc.xs_rec[cbase + c + 1]);
+        for (int32_t k = 0; k < len; k++)
+            sc.xs_rec[base + k] = value((int64_t)sc.indices[sc.xs_perm[(size_t)it.p0 + k]]);
     }
 }
 
@@ -135,16 +183,53 @@ void plan_xstage(Schedule &sc) {
     build_records(sc, kXsChunk, [&](int64_t col) {
         return sc.C == 1 ? (int32_t)xstage_stage_offset(sc.dt, (int)(col % kXsChunk)) : (int32_t)col;
     });
-    // every item's block values start on a 16-byte boundary: one bulk copy each
-    sc.xs_voff.assign(sc.items.size(), 0);
-    int64_t off = 0;
-    for (size_t i = 0; i < sc.items.size(); i++) {
-        sc.xs_voff[i] = (int32_t)std::min<int64_t>(off / 4, INT32_MAX);
-        off += xstage_pad4((int64_t)(sc.items[i].p1 - sc.items[i].p0) * sc.R * sc.C * kXsWDup);
+    const int per_block = sc.R * sc.C * kXsWDup;   // floats
+    footprints(sc, (size_t)per_block * 4, kXsChunk, kXsG, kXsTaskSizes, sc.xs.task_wbytes, sc.xs.task_ibytes);
+    // the task blobs of every task size that fits: layout, then the template
+    const int64_t n = (int64_t)sc.items.size();
+    const int64_t nch = (sc.K + kXsChunk - 1) / kXsChunk;
+    int64_t total = 0;
+    for (int gi = 0; gi < kXsTaskSizes; gi++) {
+        const int G = kXsG[gi];
+        const size_t wb = (sc.xs.task_wbytes[gi] + 15) & ~size_t(15), ib = (sc.xs.task_ibytes[gi] + 15) & ~size_t(15);
+        sc.xs_blob_off[gi] = -1;
+        if (!xstage_task_size_ok(sc.R, G) ||
+            xstage_smem_bytes(sc.dt, sc.R, sc.K, G, wb, ib) > (size_t)kXsMaxSmem)
+            continue;
+        sc.xs_blob_stride[gi] = (int64_t)G * kXsItab * 4 + (int64_t)ib + (int64_t)wb;
+        sc.xs_blob_off[gi] = (total + 255) & ~int64_t(255);
+        total = sc.xs_blob_off[gi] + (n + G - 1) / G * sc.xs_blob_stride[gi];
     }
-    sc.xs_values = off;
-    footprints(sc, (size_t)sc.R * sc.C * 4 * kXsWDup, kXsChunk, kXsG, kXsTaskSizes, sc.xs.task_wbytes,
-               sc.xs.task_ibytes);
+    sc.xs_blob.assign((size_t)(total / 4), 0);
+    sc.xs_vdst.assign((size_t)(kXsTaskSizes * n), -1);
+    for (int gi = 0; gi < kXsTaskSizes; gi++) {
+        if (sc.xs_blob_off[gi] < 0) continue;
+        const int G = kXsG[gi];
+        const int64_t ib = ((int64_t)sc.xs.task_ibytes[gi] + 15) & ~int64_t(15);
+        for (int64_t t = 0; t * G < n; t++) {
+            const int64_t blob = (sc.xs_blob_off[gi] + t * sc.xs_blob_stride[gi]) / 4;   // ints
+            const int64_t recs = blob + (int64_t)G * kXsItab, vals = recs + ib / 4;
+            int64_t woff = 0, roff = 0;
+            for (int64_t k = 0; k < G && t * G + k < n; k++) {
+                const int64_t i = t * G + k;
+                const Item &it = sc.items[(size_t)i];
+                const int64_t len = it.p1 - it.p0, rints = xstage_record_ints(len, nch);
+                int32_t *h = &sc.xs_blob[(size_t)(blob + k * kXsItab)];
+                h[0] = it.row;
+                h[1] = it.p0;
+                h[2] = it.p1;
+                h[3] = it.slot;
+                h[5] = (int32_t)len;
+                h[7] = (int32_t)woff;
+                h[8] = (int32_t)roff;
+                std::copy(sc.xs_rec.begin() + sc.xs_rec_off[(size_t)i], sc.xs_rec.begin() + sc.xs_rec_off[(size_t)i] + rints,
+                          sc.xs_blob.begin() + (recs + roff));
+                if (len) sc.xs_vdst[(size_t)(gi * n + i)] = vals + woff;
+                woff += xstage_pad4(len * per_block);
+                roff += rints;
+            }
+        }
+    }
 }
 
 void plan_tc(Schedule &sc) {
@@ -236,12 +321,14 @@ bsr_status_t build_schedule(Schedule &sc) {
         make_items(sc, limit);
         plan_xstage(sc);
     }
-    if (sc.variant == V_XSTAGE && sc.xs_values / 4 > INT32_MAX) sc.variant = V_GENERIC;   // value offsets are int32
+    if (sc.variant == V_XSTAGE && (int64_t)sc.xs_blob.size() > INT32_MAX) sc.variant = V_GENERIC;   // blob offsets are int32
     if (sc.variant == V_GENERIC) {
         sc.threads = 256;
         sc.xs_rec.clear();
         sc.xs_rec_off.clear();
-        sc.xs_voff.clear();
+        sc.xs_perm.clear();
+        sc.xs_blob.clear();
+        sc.xs_vdst.clear();
         sc.tn = std::max(1, 256 / std::min(sc.R, 256));
         make_items(sc, split_limit(sc));
     }
@@ -249,8 +336,7 @@ bsr_status_t build_schedule(Schedule &sc) {
     if (upload(&sc.d_items, sc.items) != cudaSuccess || upload(&sc.d_splits, sc.splits) != cudaSuccess ||
         upload(&sc.d_group_begin, sc.group_begin) != cudaSuccess ||
         upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess ||
-        upload(&sc.d_xs_rec, sc.xs_rec) != cudaSuccess || upload(&sc.d_xs_rec_off, sc.xs_rec_off) != cudaSuccess ||
-        upload(&sc.d_xs_voff, sc.xs_voff) != cudaSuccess) {
+        upload(&sc.d_xs_perm, sc.xs_perm) != cudaSuccess || upload(&sc.d_xs_vdst, sc.xs_vdst) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
@@ -266,17 +352,26 @@ bsr_status_t build_schedule(Schedule &sc) {
 bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
     const Schedule &sc = *h.sched;
-    if ((sc.variant != V_XSTAGE && sc.variant != V_TC) || sc.nnzb == 0) return BSR_OK;
-    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * sc.R * sc.C * 2 : (size_t)sc.xs_values * 4;
+    if (sc.variant == V_TC && sc.nnzb == 0) return BSR_OK;
+    if (sc.variant != V_XSTAGE && sc.variant != V_TC) return BSR_OK;
+    // xstage: the task blobs (item tables and records from the schedule's
+    // template, then this handle's block values)
+    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * sc.R * sc.C * 2 : sc.xs_blob.size() * 4;
+    if (bytes == 0) return BSR_OK;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
         h.data_packed = nullptr;
         return BSR_ERR_ALLOC;
     }
-    cudaError_t e = sc.variant == V_TC
-                        ? pack_tc_data(h.data, sc.nnzb, sc.R, sc.C, (uint16_t *)h.data_packed, 0)
-                        : pack_xstage_data(h.data, sc.dt, sc.d_items, sc.d_xs_voff, (int64_t)sc.items.size(), sc.R,
-                                           sc.C, (float *)h.data_packed, 0);
+    cudaError_t e = cudaSuccess;
+    if (sc.variant == V_TC) {
+        e = pack_tc_data(h.data, sc.nnzb, sc.R, sc.C, (uint16_t *)h.data_packed, 0);
+    } else {
+        e = cudaMemcpy(h.data_packed, sc.xs_blob.data(), bytes, cudaMemcpyHostToDevice);
+        if (e == cudaSuccess && sc.nnzb > 0)
+            e = pack_xstage_data(h.data, sc.dt, sc.d_items, sc.d_xs_perm, sc.d_xs_vdst, (int64_t)sc.items.size(),
+                                 sc.R, sc.C, (float *)h.data_packed, 0);
+    }
     if (e != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_CUDA;
@@ -297,12 +392,7 @@ int choose_tasks(const Schedule &sc, int64_t N) {
         const char *v = getenv("BSR_XS_G");
         return v ? atoi(v) : 0;
     }();
-    auto fits = [&](int G) {
-        const int gi = g_index(G);
-        return xstage_task_size_ok(sc.R, G) &&
-               xstage_smem_bytes(sc.dt, sc.R, sc.K, G, sc.xs.task_wbytes[gi], sc.xs.task_ibytes[gi]) <=
-                   (size_t)kXsMaxSmem;
-    };
+    auto fits = [&](int G) { return sc.xs_blob_off[g_index(G)] >= 0; };   // blobs exist for G
     for (int gi = 0; gi < kXsTaskSizes; gi++)
         if (forced == kXsG[gi] && fits(forced)) return forced;
     const double kFixed = 10000.0;

@@ -58,7 +58,7 @@ constexpr int NS = kXsStages;
 constexpr int NCW = kXsConsumerWarps;
 constexpr int NTHREADS = (NCW + 1) * 32;
 constexpr int WD = kXsWDup;
-constexpr int kItab = 12;  // ints per item in the shared item table
+constexpr int kItab = kXsItab;   // ints per item in a task's item table
 #ifndef XS_UNROLL
 #define XS_UNROLL 1
 #endif
@@ -66,19 +66,16 @@ constexpr int kUnroll = XS_UNROLL;   // unrolling of the one-column block loop
 constexpr uint64_t kDrainNs = 200000000ull;   // bound for TMA loads already issued (they take microseconds)
 
 struct XsArgs {
-    const Item *items;
     int n_items, G, S, n_tasks;
-    const int32_t *rec;      // per-item records (xstage_record_ints)
-    const int32_t *rec_off;  // per item: record offset in ints
-    const float *wpk;        // per item, 16-byte aligned: [block][C][R][WD]
+    const unsigned char *blob;   // task t's blob at blob + t * stride (see xstage.h)
+    uint32_t stride, hdr, ib;    // blob bytes per task, item-table bytes, record-region bytes
     const float *bias;
     void *Y;
     float *ws;
     int *status;
     int64_t N, K, M;
     int C, nchunks;
-    uint32_t w_off, idx_off, bias_off, bar_off, misc_off;
-    const int32_t *voff;     // per item: offset of its packed values in 16-byte units
+    uint32_t blob_off, bias_off, bar_off, misc_off;   // shared-memory offsets
     uint64_t wait_ns;
     int stall_chunk;         // test hook: this chunk is never loaded (-1: none)
 };
@@ -206,8 +203,8 @@ __device__ __forceinline__ bool aborted(const int *flag) {
 struct Shared {
     unsigned char *base;
     uint64_t *full, *empty;
-    int *misc;          // [0] abort flag
-    int *itab;          // per item (kItab ints): row p0 p1 slot rec_off len voff16 woff roff
+    int *misc;          // [0] abort flag, [3] task covers consecutive whole rows
+    int *itab;          // the blob's item table (kItab ints per item)
     float *W;           // block values of the task's items
     int32_t *I;         // the task's item records
     float *B;           // [item][R] bias
@@ -223,15 +220,15 @@ __device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *s
     constexpr int NKS = 4 / NRG;
     constexpr int R = TR * NRG;
     const int lo = cb[c], hi = cb[c + 1];
-    int j0 = lo, j1 = hi;
-    if (S > 1) {
-        j0 = lo <= piece ? 0 : (lo - piece + S - 1) / S;
-        j1 = hi <= piece ? 0 : (hi - piece + S - 1) / S;
-    }
     if constexpr (CT == 1) {
+        // groups of NKS consecutive blocks (ordered on the host so that a
+        // group's columns fall in distinct banks), dealt round-robin to the
+        // S warps of the item; lane group ks takes block ks of each group
+        const int ngr = (hi - lo + NKS - 1) / NKS;
 #pragma unroll kUnroll
-        for (int jj = j0 + ks; jj < j1; jj += NKS) {
-            const int lb = piece + S * jj;
+        for (int jg = piece; jg < ngr; jg += S) {
+            const int lb = lo + jg * NKS + ks;
+            if (NKS > 1 && lb >= hi) continue;
             const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
             float x[8];
             f2_t wd[TR];
@@ -240,11 +237,17 @@ __device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *s
             load_wd<TR>(wbase + lb * R * WD, wd);
             acc.fma(x, wd);
         }
+        return;
     } else {
         // wide blocks (a multiple of 4 columns per lane group): the NKS lane
         // groups split each block's columns, so no lanes idle when a chunk
         // holds fewer blocks than groups; narrow blocks: groups take
         // alternate blocks
+        int j0 = lo, j1 = hi;
+        if (S > 1) {
+            j0 = lo <= piece ? 0 : (lo - piece + S - 1) / S;
+            j1 = hi <= piece ? 0 : (hi - piece + S - 1) / S;
+        }
         const int kbase = c * KC;
         const bool csplit = NKS > 1 && C % (4 * NKS) == 0;
         const int cw = csplit ? C / NKS : C;
@@ -347,7 +350,7 @@ __device__ __forceinline__ void store_tile(const XsArgs &a, const Shared &sh, co
 // and a pairwise tree sums them. RW > 1 (G = 12 RW): each warp owns RW
 // whole items, with one register tile each, and needs no tree.
 template <typename T, int TR, int NRG, int CT, int RW>
-__device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int64_t n0, int item_first,
+__device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int64_t n0, int task,
                                          int g_count, uint32_t CL, int warp, int lane) {
     using St = Stage<T>;
     constexpr int R = TR * NRG;
@@ -355,42 +358,27 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     const int nch = a.nchunks;
     const int ctid = threadIdx.x;   // 0 .. NCW*32-1
 
-    // ---- each item's shared-memory offsets, then the task's block values
-    // and records (consecutive in memory: the task's items are consecutive)
-    // by 16-byte asynchronous copies from all consumer threads, and the bias
-    if (ctid < g_count) {
-        int woff = 0, roff = 0;
-        for (int k = 0; k <= ctid; k++) {
-            const int len = sh.itab[kItab * k + 5];
-            if (k == ctid) {
-                sh.itab[kItab * k + 7] = woff;
-                sh.itab[kItab * k + 8] = roff;
-            }
-            woff += (int)xstage_pad4((int64_t)len * R * C * WD);
-            roff += (int)xstage_record_ints(len, nch);
-        }
-        if (ctid == g_count - 1) {
-            sh.misc[1] = woff;   // floats
-            sh.misc[2] = roff;   // ints
-        }
-        // does the task cover consecutive whole rows? (then the epilogue
-        // stores whole row segments of Y)
-        if (sh.itab[kItab * ctid + 0] != sh.itab[0] + ctid || sh.itab[kItab * ctid + 3] >= 0) sh.misc[3] = 0;
-    }
-    ptx::named_barrier(1, NCW * 32);
+    // ---- the task's blob (item table, records, block values) in one round
+    // trip: 16-byte asynchronous copies from all consumer threads
     if (g_count > 0) {
-        const int wq = sh.misc[1] / 4, rq = sh.misc[2] / 4;   // 16-byte pieces
-        const float4 *ws = reinterpret_cast<const float4 *>(a.wpk + (int64_t)sh.itab[6] * 4);
-        const int4 *rs = reinterpret_cast<const int4 *>(a.rec + sh.itab[4]);
-        for (int e = ctid; e < wq; e += NCW * 32) ptx::cp_async16(reinterpret_cast<float4 *>(sh.W) + e, ws + e);
-        for (int e = ctid; e < rq; e += NCW * 32) ptx::cp_async16(reinterpret_cast<int4 *>(sh.I) + e, rs + e);
-    }
-    for (int e = ctid; e < g_count * R; e += NCW * 32) {   // one bias value per thread: loads in parallel
-        const int g = e / R, r = e - g * R;
-        sh.B[e] = a.bias ? __ldg(a.bias + (int64_t)sh.itab[kItab * g + 0] * R + r) : 0.f;
+        const int4 *src = reinterpret_cast<const int4 *>(a.blob + (int64_t)task * a.stride);
+        int4 *dst = reinterpret_cast<int4 *>(sh.itab);
+        for (int e = ctid; e < (int)(a.stride / 16); e += NCW * 32) ptx::cp_async16(dst + e, src + e);
     }
     ptx::cp_async_wait_all();
     ptx::named_barrier(1, NCW * 32);
+    // the bias, needed only by the epilogue (waited for there), and whether
+    // the task covers consecutive whole rows (then the epilogue stores whole
+    // row segments of Y)
+    for (int e = ctid; e < g_count * R; e += NCW * 32) {
+        const int g = e / R, r = e - g * R;
+        if (a.bias)
+            ptx::cp_async4(&sh.B[e], a.bias + (int64_t)sh.itab[kItab * g + 0] * R + r);
+        else
+            sh.B[e] = 0.f;
+    }
+    if (ctid < g_count && (sh.itab[kItab * ctid + 0] != sh.itab[0] + ctid || sh.itab[kItab * ctid + 3] >= 0))
+        sh.misc[3] = 0;
     bool ok = true;
 
     const int q = lane >> 3, tg = lane & 7;
@@ -428,6 +416,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
             set_status(a.status, DEV_TIMEOUT);
             atomicExch(&sh.misc[0], 1);
         }
+        ptx::cp_async_wait_all();   // the bias
         if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
         if (R == 1 && sh.misc[3]) {
             // consecutive rows row0 .. row0+G-1: transpose the tiles through
@@ -495,6 +484,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     reduce_tile<TR, NRG>(acc, v);
     // every consumer is done with the ring and the block values; the abort
     // verdict is the same for all of them (barrier reduction)
+    ptx::cp_async_wait_all();   // the bias
     if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
     // pairwise tree over the S warps of each item: in round `step`, the warp
     // of piece p (p % 2step == step) hands its tile to piece p - step
@@ -554,9 +544,9 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     sh.full = reinterpret_cast<uint64_t *>(sh.base + a.bar_off);
     sh.empty = sh.full + NS;
     sh.misc = reinterpret_cast<int *>(sh.base + a.misc_off);
-    sh.itab = sh.misc + 4;
-    sh.W = reinterpret_cast<float *>(sh.base + a.w_off);
-    sh.I = reinterpret_cast<int32_t *>(sh.base + a.idx_off);
+    sh.itab = reinterpret_cast<int *>(sh.base + a.blob_off);
+    sh.I = reinterpret_cast<int32_t *>(sh.base + a.blob_off + a.hdr);
+    sh.W = reinterpret_cast<float *>(sh.base + a.blob_off + a.hdr + a.ib);
     sh.B = reinterpret_cast<float *>(sh.base + a.bias_off);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -580,17 +570,6 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
         sh.misc[0] = 0;
         sh.misc[3] = 1;
         ptx::fence_barrier_init();
-    }
-    if ((int)threadIdx.x < g_count) {   // one thread per item fills the item table
-        const int g = threadIdx.x;
-        const Item it = a.items[item_first + g];
-        sh.itab[kItab * g + 0] = it.row;
-        sh.itab[kItab * g + 1] = it.p0;
-        sh.itab[kItab * g + 2] = it.p1;
-        sh.itab[kItab * g + 3] = it.slot;
-        sh.itab[kItab * g + 4] = __ldg(a.rec_off + item_first + g);
-        sh.itab[kItab * g + 5] = it.p1 - it.p0;
-        sh.itab[kItab * g + 6] = __ldg(a.voff + item_first + g);
     }
     // every CTA's barriers exist before any multicast or remote arrive
     if (CL == 1) __syncthreads(); else ptx::cluster_sync();
@@ -630,28 +609,31 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
         }
         __syncwarp();
     } else {
-        consumer<T, TR, NRG, CT, RW>(a, sh, n0, item_first, g_count, CL, warp, lane);
+        consumer<T, TR, NRG, CT, RW>(a, sh, n0, task, g_count, CL, warp, lane);
     }
     if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
 }
 
-// Block values in the kernel's layout: item by item (each item starting on a
-// 16-byte boundary), per block W^T widened to fp32 with WD copies of each
-// value: wpk[4*voff[i] + ((b*C + c)*R + r)*WD + d] = data[((p0_i + b)*R + r)*C + c].
+// Block values into the task blobs of every task size: item i's values go to
+// blobs + vdst[g * n_items + i] (floats; -1: none), blocks in the records'
+// order (perm: position -> stored block), per block W^T widened to fp32
+// with WD copies: [(b*C + c)*R + r]*WD + d <- data[(perm[p0_i + b]*R + r)*C + c].
 template <typename T>
-__global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ items, const int32_t *__restrict__ voff,
-                       int64_t n_items, float *__restrict__ wpk, int R, int C) {
-    for (int64_t i = blockIdx.x; i < n_items; i += gridDim.x) {
-        const Item it = items[i];
+__global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ items, const int32_t *__restrict__ perm,
+                       const int64_t *__restrict__ vdst, int64_t n_items, float *__restrict__ blobs, int R, int C) {
+    for (int64_t gi = blockIdx.x; gi < kXsTaskSizes * n_items; gi += gridDim.x) {
+        const int64_t d = vdst[gi];
+        if (d < 0) continue;
+        const Item it = items[gi % n_items];
         const int64_t total = (int64_t)(it.p1 - it.p0) * R * C;
-        float *dst = wpk + 4 * (int64_t)voff[i];
+        float *dst = blobs + d;
         for (int64_t e = threadIdx.x; e < total; e += blockDim.x) {
             const int64_t b = e / ((int64_t)R * C);
             const int rc = (int)(e - b * R * C);
             const int c = rc / R, r = rc - c * R;
-            const float w = to_f32(data[((it.p0 + b) * R + r) * C + c]);
+            const float w = to_f32(data[((int64_t)perm[it.p0 + b] * R + r) * C + c]);
 #pragma unroll
-            for (int d = 0; d < WD; d++) dst[WD * e + d] = w;
+            for (int k = 0; k < WD; k++) dst[WD * e + k] = w;
         }
     }
 }
@@ -732,15 +714,16 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     auto enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
 
+    if (sc.xs_blob_off[gidx] < 0 || la.data == nullptr) return cudaErrorInvalidConfiguration;
     XsArgs a;
-    a.items = sc.d_items;
     a.n_items = n_items;
     a.G = G;
     a.S = G <= NCW ? NCW / G : 1;
     a.n_tasks = (n_items + G - 1) / G;
-    a.rec = sc.d_xs_rec;
-    a.rec_off = sc.d_xs_rec_off;
-    a.wpk = static_cast<const float *>(la.data);
+    a.blob = static_cast<const unsigned char *>(la.data) + sc.xs_blob_off[gidx];
+    a.stride = (uint32_t)sc.xs_blob_stride[gidx];
+    a.hdr = (uint32_t)(G * kItab * 4);
+    a.ib = (uint32_t)((pl.task_ibytes[gidx] + 15) & ~size_t(15));
     a.bias = la.bias;
     a.Y = la.Y;
     a.ws = la.ws;
@@ -750,13 +733,11 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.M = sc.M;
     a.C = sc.C;
     a.nchunks = (int)((sc.K + KC - 1) / KC);
-    a.w_off = (uint32_t)region_bytes(sc.dt, sc.R);
-    a.idx_off = a.w_off + (uint32_t)((pl.task_wbytes[gidx] + 15) & ~size_t(15));
-    a.bias_off = a.idx_off + (uint32_t)((pl.task_ibytes[gidx] + 15) & ~size_t(15));
+    a.blob_off = (uint32_t)region_bytes(sc.dt, sc.R);
+    a.bias_off = a.blob_off + a.stride;
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * sc.R * 4 + 15) & ~size_t(15));
     a.misc_off = a.bar_off + (2 * NS + 1) * 8;
-    a.voff = sc.d_xs_voff;
-    const uint32_t smem = a.misc_off + (4 + kItab * G) * 4 + 1024;   // + slack to align the base
+    const uint32_t smem = a.misc_off + 4 * 4 + 1024;   // + slack to align the base
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
     static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
@@ -847,10 +828,9 @@ cudaError_t launch_r(const LaunchArgs &la, const XsPlan &pl, int G) {
 }  // namespace
 
 size_t xstage_smem_bytes(bsr_dtype_t dt, int R, int64_t K, int G, size_t wbytes, size_t ibytes) {
-    const size_t nch = (size_t)((K + KC - 1) / KC);
-    (void)nch;
-    return region_bytes(dt, R) + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + (4 + kItab * (size_t)G) * 4 + 1024;
+    (void)K;
+    return region_bytes(dt, R) + (size_t)G * kItab * 4 + ((wbytes + 15) & ~size_t(15)) +
+           ((ibytes + 15) & ~size_t(15)) + (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 1) * 8 + 4 * 4 + 1024;
 }
 
 size_t xstage_task_budget(bsr_dtype_t dt, int R, int64_t K) {
@@ -877,14 +857,14 @@ bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
     return r_ok && c_ok && K % align == 0 && K > 0;
 }
 
-cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *voff,
-                             int64_t n_items, int R, int C, float *wpk, cudaStream_t s) {
+cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
+                             const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s) {
     if (n_items == 0) return cudaSuccess;
-    const int grid = (int)std::min<int64_t>(n_items, 1 << 16);
+    const int grid = (int)std::min<int64_t>(kXsTaskSizes * n_items, 1 << 16);
     if (dt == BSR_F32)
-        k_pack<float><<<grid, 256, 0, s>>>((const float *)data, items, voff, n_items, wpk, R, C);
+        k_pack<float><<<grid, 256, 0, s>>>((const float *)data, items, perm, vdst, n_items, blobs, R, C);
     else
-        k_pack<uint16_t><<<grid, 256, 0, s>>>((const uint16_t *)data, items, voff, n_items, wpk, R, C);
+        k_pack<uint16_t><<<grid, 256, 0, s>>>((const uint16_t *)data, items, perm, vdst, n_items, blobs, R, C);
     return cudaGetLastError();
 }
 

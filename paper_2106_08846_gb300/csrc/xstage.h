@@ -21,8 +21,17 @@ constexpr int kXsWDup = 1;             // copies of each packed block value
 constexpr int kXsTaskSizes = 8;
 constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12, 24, 48};
 
+constexpr int kXsItab = 12;   // ints per item in a task's item table
+
 // Per task size (index into kXsG): the largest shared-memory footprint of
 // block values / indices over all tasks of G consecutive items.
+//
+// Everything one task needs is one contiguous "blob" in device memory, at a
+// fixed stride per task size, so a CTA fetches it in one round trip without
+// first reading any table: [ item table: G x kXsItab ints (row, p0, p1,
+// slot, -, len, -, woff, roff, -, -, -) | records (task_ibytes, 16-byte
+// padded) | block values (task_wbytes, 16-byte padded) ]. woff (floats) and
+// roff (ints) locate an item's values and record inside their regions.
 struct XsPlan {
     size_t task_wbytes[kXsTaskSizes] = {};
     size_t task_ibytes[kXsTaskSizes] = {};   // item records (see xstage_record_ints)
