@@ -128,7 +128,7 @@ struct LaunchArgs {
 cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
-cudaError_t pack_tc_data(const void *data, int64_t nnzb, int R, int C, uint16_t *out, cudaStream_t s);
+cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, void *out, cudaStream_t s);
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
                              const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);

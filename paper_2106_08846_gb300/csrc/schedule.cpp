@@ -233,8 +233,10 @@ void plan_xstage(Schedule &sc) {
 }
 
 void plan_tc(Schedule &sc) {
-    const int64_t nch = (sc.K + kTcChunk - 1) / kTcChunk;
-    const size_t per_block = (size_t)sc.R * sc.C * 2;
+    const int kc = tc_chunk_cols(sc.dt);
+    const int64_t es = (int64_t)dtype_size(sc.dt);
+    const int64_t nch = (sc.K + kc - 1) / kc;
+    const size_t per_block = tc_block_bytes(sc.R, sc.C, sc.dt);
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         const int G = kTcG[gi];
         std::vector<int32_t> &rec = sc.tc.rec[gi];
@@ -251,8 +253,8 @@ void plan_tc(Schedule &sc) {
                 const Item &it = sc.items[k];
                 for (int32_t b = 0; b < it.p1 - it.p0; b++) {
                     const int64_t col = sc.indices[it.p0 + b];
-                    const int64_t c = (col * sc.C) / kTcChunk;
-                    const int32_t a32 = (int32_t)(((col * sc.C) % kTcChunk) * 2 / 32);
+                    const int64_t c = (col * sc.C) / kc;
+                    const int32_t a32 = (int32_t)(((col * sc.C) % kc) * es / 32);
                     per_chunk[(size_t)c].push_back(a32 | (int32_t)((k - t) << 2) | ((b == 0) << 7) |
                                                    ((wblk + b) << 8));
                 }
@@ -300,9 +302,9 @@ bsr_status_t build_schedule(Schedule &sc) {
         sc.variant = V_TC;
         sc.tn = kTcTokens;
         sc.threads = 192;
-        const int64_t nch = (sc.K + kTcChunk - 1) / kTcChunk;
-        const int64_t avail = (int64_t)tc_task_budget(sc.R) - 4 * xstage_pad4(nch + 1) - 16;
-        const int64_t lmax = std::max<int64_t>(1, avail / (int64_t)((size_t)sc.R * sc.C * 2 + 4));
+        const int64_t nch = (sc.K + tc_chunk_cols(sc.dt) - 1) / tc_chunk_cols(sc.dt);
+        const int64_t avail = (int64_t)tc_task_budget(sc.R, sc.dt) - 4 * xstage_pad4(nch + 1) - 16;
+        const int64_t lmax = std::max<int64_t>(1, avail / (int64_t)(tc_block_bytes(sc.R, sc.C, sc.dt) + 4));
         int64_t limit = split_limit(sc);
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
         make_items(sc, limit);
@@ -356,7 +358,7 @@ bsr_status_t pack_data(Handle &h) {
     if (sc.variant != V_XSTAGE && sc.variant != V_TC) return BSR_OK;
     // xstage: the task blobs (item tables and records from the schedule's
     // template, then this handle's block values)
-    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * sc.R * sc.C * 2 : sc.xs_blob.size() * 4;
+    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * tc_block_bytes(sc.R, sc.C, sc.dt) : sc.xs_blob.size() * 4;
     if (bytes == 0) return BSR_OK;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
@@ -365,7 +367,7 @@ bsr_status_t pack_data(Handle &h) {
     }
     cudaError_t e = cudaSuccess;
     if (sc.variant == V_TC) {
-        e = pack_tc_data(h.data, sc.nnzb, sc.R, sc.C, (uint16_t *)h.data_packed, 0);
+        e = pack_tc_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, h.data_packed, 0);
     } else {
         e = cudaMemcpy(h.data_packed, sc.xs_blob.data(), bytes, cudaMemcpyHostToDevice);
         if (e == cudaSuccess && sc.nnzb > 0)
@@ -425,7 +427,7 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
     auto fits = [&](int G) {
         const int gi = tc_g_index(G);
         return G * sc.R <= kTcTmemCols &&
-               tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi]) <= (size_t)kTcMaxSmem;
+               tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt) <= (size_t)kTcMaxSmem;
     };
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (forced == kTcG[gi] && fits(forced)) return forced;

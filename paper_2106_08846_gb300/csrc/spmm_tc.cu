@@ -40,9 +40,15 @@ namespace bsr {
 namespace {
 
 constexpr int TN = kTcTokens;
-constexpr int KC = kTcChunk;
-constexpr int NS = kTcStages;
-constexpr uint32_t kStageBytes = TN * KC * 2;   // 16 KB: 128 rows of 128 bytes
+constexpr uint32_t kStageBytes = TN * 128;   // 16 KB: 128 token rows of 128 bytes (64 bf16 or 32 fp32 columns)
+constexpr int kMaxStages = kTcStages;
+// Per element type: K columns per stage and ring depth (fp32 stages come
+// with a second buffer holding the low parts of the split operand).
+template <typename T>
+struct TcCfg {
+    static constexpr int KC = 128 / (int)sizeof(T);
+    static constexpr int NS = sizeof(T) == 4 ? kTcStagesF32 : kTcStages;
+};
 constexpr int NWARPS = 6;
 constexpr int NTHREADS = NWARPS * 32;
 constexpr uint64_t kDrainNs = 200000000ull;
@@ -52,9 +58,9 @@ struct TcArgs {
     int n_items, G, n_tasks;
     const int32_t *trec;      // task records: chunk starts, then MMA entries
     const int32_t *trec_off;  // per task: record offset (ints)
-    const uint16_t *wpk;      // block values in the MMA's B layout
+    const void *wpk;          // block values in the MMA's B layout (fp32: high then low parts)
     const float *bias;
-    uint16_t *Y;
+    void *Y;
     float *ws;
     int *status;
     int64_t N, K, M;
@@ -85,6 +91,25 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b
         "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
         ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc));
+}
+
+// Instruction descriptor of kind::tf32: tf32 A and B (format 2), fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
+    return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc));
+}
+
+// fp32 -> (high, low) with high = x with the low 13 mantissa bits cleared
+// (a tf32 value) and low = x - high, exact in fp32.
+__device__ __forceinline__ float4 tf32_high(float4 v) {
+    return make_float4(__uint_as_float(__float_as_uint(v.x) & 0xffffe000u), __uint_as_float(__float_as_uint(v.y) & 0xffffe000u),
+                       __uint_as_float(__float_as_uint(v.z) & 0xffffe000u), __uint_as_float(__float_as_uint(v.w) & 0xffffe000u));
 }
 
 // The mbarrier arrives once every MMA this thread issued so far completed.
@@ -127,15 +152,18 @@ __device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[3
         : "r"(taddr));
 }
 
-template <int R>
+template <typename T, int R>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
+    constexpr bool F32 = sizeof(T) == 4;
+    constexpr int NS = TcCfg<T>::NS;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base =
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(base + a.bar_off);
     uint64_t *empty = full + NS;
-    uint64_t *wbar = empty + NS;     // block values landed
+    uint64_t *split = empty + NS;    // fp32: the stage's high/low parts are ready
+    uint64_t *wbar = split + NS;     // block values landed
     uint64_t *done = wbar + 1;       // every MMA completed
     uint64_t *rbar = done + 1;       // task record landed
     int *misc = reinterpret_cast<int *>(base + a.misc_off);   // [0] abort flag, [1] TMEM address
@@ -156,6 +184,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         for (int s = 0; s < NS; s++) {
             ptx::mbar_init(&full[s], 1);
             ptx::mbar_init(&empty[s], 1);
+            ptx::mbar_init(&split[s], 1);
         }
         ptx::mbar_init(wbar, 1);
         ptx::mbar_init(done, 1);
@@ -184,6 +213,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = (uint32_t)misc[1];
+    const uint32_t wblock = (uint32_t)R * C * (F32 ? 8 : 2);   // bytes of one block's B operand(s)
 
     if (warp == 0) {
         // ---------------- producer
@@ -194,14 +224,14 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
             const uint32_t rec_bytes = (uint32_t)(pad4(nch + 1) + pad4(n_ent)) * 4;
             ptx::mbar_arrive_expect_tx(rbar, rec_bytes);
             ptx::bulk_load(I_s, trec, rec_bytes, rbar);
-            const uint32_t wblock = (uint32_t)R * C * 2;
             uint32_t total = 0;
             for (int g = 0; g < g_count; g++) total += (uint32_t)itab[6 * g + 5] * wblock;
             ptx::mbar_arrive_expect_tx(wbar, total);
             uint32_t woff = 0;
+            const unsigned char *wsrc = static_cast<const unsigned char *>(a.wpk);
             for (int g = 0; g < g_count; g++) {
                 const int len = itab[6 * g + 5];
-                if (len) ptx::bulk_load(W_s + woff, a.wpk + (int64_t)itab[6 * g + 1] * R * C, len * wblock, wbar);
+                if (len) ptx::bulk_load(W_s + woff, wsrc + (int64_t)itab[6 * g + 1] * wblock, len * wblock, wbar);
                 woff += len * wblock;
             }
             int k = 0;          // ring slots used (chunks with work, in order)
@@ -220,7 +250,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                     continue;
                 }
                 ptx::mbar_arrive_expect_tx(&full[s], kStageBytes);
-                ptx::tma_load_2d(base + s * kStageBytes, &xmap, c * KC, (int32_t)n0, &full[s]);
+                ptx::tma_load_2d(base + s * kStageBytes, &xmap, c * TcCfg<T>::KC, (int32_t)n0, &full[s]);
                 k++;
             }
             if (!ok) {
@@ -235,7 +265,6 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
     } else if (warp == 1) {
         // ---------------- MMA issuer
         if (lane == 0) {
-            constexpr uint32_t idesc = idesc_bf16(TN, R);
             bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns) && ptx::mbar_wait_bounded(wbar, 0, a.wait_ns) &&
                       !aborted(misc);
             const uint32_t w_base = ptx::smem_addr(W_s);
@@ -245,7 +274,8 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                 const int lo = I_s[c], hi = I_s[c + 1];
                 if (lo == hi) continue;
                 const int s = k % NS;
-                if (!ptx::mbar_wait_bounded(&full[s], (k / NS) & 1, a.wait_ns) || aborted(misc)) {
+                // fp32: wait for the split parts (the split warps waited for the copy)
+                if (!ptx::mbar_wait_bounded(F32 ? &split[s] : &full[s], (k / NS) & 1, a.wait_ns) || aborted(misc)) {
                     ok = false;
                     break;
                 }
@@ -255,12 +285,29 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                     const uint32_t v = (uint32_t)ent[e];
                     const uint32_t a_row = stage + (v & 3u) * 32u;
                     const uint32_t g = (v >> 2) & 31u, first = (v >> 7) & 1u;
-                    const uint32_t w_blk = w_base + (v >> 8) * (uint32_t)(R * C * 2);
+                    const uint32_t w_blk = w_base + (v >> 8) * wblock;
+                    if constexpr (F32) {
+                        // 3xTF32: high x high + high x low + low x high, K = 8 per MMA
+                        constexpr uint32_t idesc = idesc_tf32(TN, R);
+                        const uint32_t a_lo = a_row + NS * kStageBytes, w_lo = w_blk + (uint32_t)R * C * 4;
+#pragma unroll 2
+                        for (int sl = 0; sl < C / 8; sl++) {
+                            const uint64_t ah = umma_desc(a_row + sl * 32, 16, 1024, 2);
+                            const uint64_t al = umma_desc(a_lo + sl * 32, 16, 1024, 2);
+                            const uint64_t bh = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
+                            const uint64_t bl = umma_desc(w_lo + sl * (R * 32), 128, 256, 0);
+                            mma_tf32(tmem + g * R, ah, bh, idesc, (first == 0u) | (sl > 0));
+                            mma_tf32(tmem + g * R, ah, bl, idesc, 1u);
+                            mma_tf32(tmem + g * R, al, bh, idesc, 1u);
+                        }
+                    } else {
+                        constexpr uint32_t idesc = idesc_bf16(TN, R);
 #pragma unroll 4
-                    for (int sl = 0; sl < C / 16; sl++) {
-                        const uint64_t ad = umma_desc(a_row + sl * 32, 16, 1024, 2);
-                        const uint64_t bd = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
-                        mma_bf16(tmem + g * R, ad, bd, idesc, (first == 0u) | (sl > 0));
+                        for (int sl = 0; sl < C / 16; sl++) {
+                            const uint64_t ad = umma_desc(a_row + sl * 32, 16, 1024, 2);
+                            const uint64_t bd = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
+                            mma_bf16(tmem + g * R, ad, bd, idesc, (first == 0u) | (sl > 0));
+                        }
                     }
                 }
                 mma_commit(&empty[s]);   // the stage is free once these MMAs completed
@@ -273,18 +320,50 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
             mma_commit(done);   // every MMA issued above completes before `done`
         }
     } else {
-        // ---------------- epilogue: warps 2..5, TMEM lane quarter = warp % 4
+        // ---------------- warps 2..5: fp32 split during the main loop, then
+        // the epilogue; TMEM lane quarter = warp % 4
         const int et = threadIdx.x - 64;   // 0..127
         for (int e = et; e < g_count * R; e += 128) {
             const int g = e / R, r = e - g * R;
             B_s[e] = a.bias ? __ldg(a.bias + (int64_t)itab[6 * g + 0] * R + r) : 0.f;
+        }
+        bool split_ok = true;
+        if constexpr (F32) {
+            // x = high + low per element of every loaded stage: high in
+            // place, low into the stage's twin buffer (same swizzled layout)
+            split_ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);
+            int k = 0;
+            for (int c = 0; split_ok && c < nch; c++) {
+                if (I_s[c] == I_s[c + 1]) continue;
+                const int s = k % NS;
+                const bool got = ptx::mbar_wait_bounded(&full[s], (k / NS) & 1, a.wait_ns) && !aborted(misc);
+                if (ptx::named_barrier_or(2, 128, !got)) { split_ok = false; break; }
+                float4 *hi4 = reinterpret_cast<float4 *>(base + s * kStageBytes);
+                float4 *lo4 = reinterpret_cast<float4 *>(base + (NS + s) * kStageBytes);
+#pragma unroll
+                for (int j = 0; j < (int)(kStageBytes / 16 / 128); j++) {
+                    const int q4 = et + 128 * j;
+                    const float4 x = hi4[q4];
+                    const float4 h = tf32_high(x);
+                    hi4[q4] = h;
+                    lo4[q4] = make_float4(x.x - h.x, x.y - h.y, x.z - h.z, x.w - h.w);
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the tensor cores
+                ptx::named_barrier(2, 128);
+                if (et == 0) ptx::mbar_arrive(&split[s]);
+                k++;
+            }
+            if (!split_ok && et == 0) {
+                set_status(a.status, DEV_TIMEOUT);
+                atomicExch(&misc[0], 1);
+            }
         }
         ptx::named_barrier(1, 128);
         // the last commit fires after the whole main loop: allow it every chunk's bound
         const uint64_t limit = a.wait_ns * (uint64_t)(nch + 2);
         const bool got = ptx::mbar_wait_bounded(done, 0, limit);
         tc_fence_after();
-        const bool stop = ptx::named_barrier_or(1, 128, !got || aborted(misc));
+        const bool stop = ptx::named_barrier_or(1, 128, !got || !split_ok || aborted(misc));
         if (!got && et == 0) set_status(a.status, DEV_TIMEOUT);
         const int q = warp & 3;
         const int64_t n = n0 + 32 * q + lane;
@@ -306,16 +385,24 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
 #pragma unroll
                 for (int j = 0; j < 16; j++) v[j] = len > 0 ? __uint_as_float(h < 32 ? r0[h + j] : r1[h - 32 + j]) : 0.f;
                 if (slot < 0) {
-                    uint32_t pk[8];
+                    if constexpr (F32) {
+                        float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.Y) + n * a.M + (int64_t)row * R + hr);
 #pragma unroll
-                    for (int j = 0; j < 8; j++) {
-                        const float lo = v[2 * j] + B_s[col + 2 * j];
-                        const float hi = v[2 * j + 1] + B_s[col + 2 * j + 1];
-                        pk[j] = (uint32_t)from_f32<uint16_t>(lo) | ((uint32_t)from_f32<uint16_t>(hi) << 16);
+                        for (int j = 0; j < 4; j++)
+                            dst[j] = make_float4(v[4 * j] + B_s[col + 4 * j], v[4 * j + 1] + B_s[col + 4 * j + 1],
+                                                 v[4 * j + 2] + B_s[col + 4 * j + 2], v[4 * j + 3] + B_s[col + 4 * j + 3]);
+                    } else {
+                        uint32_t pk[8];
+#pragma unroll
+                        for (int j = 0; j < 8; j++) {
+                            const float lo = v[2 * j] + B_s[col + 2 * j];
+                            const float hi = v[2 * j + 1] + B_s[col + 2 * j + 1];
+                            pk[j] = (uint32_t)from_f32<uint16_t>(lo) | ((uint32_t)from_f32<uint16_t>(hi) << 16);
+                        }
+                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<uint16_t *>(a.Y) + n * a.M + (int64_t)row * R + hr);
+                        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                     }
-                    uint4 *dst = reinterpret_cast<uint4 *>(a.Y + n * a.M + (int64_t)row * R + hr);
-                    dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                    dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                 } else {
                     float4 *dst = reinterpret_cast<float4 *>(a.ws + ((int64_t)slot * a.N + n) * R + hr);
 #pragma unroll
@@ -349,6 +436,23 @@ __global__ void k_pack_tc(const uint16_t *__restrict__ data, uint16_t *__restric
     }
 }
 
+// fp32 block values as two tf32 B operands, high part then low part, each in
+// the layout above with 8-column K-slices of 8-row x 16-byte core matrices.
+__global__ void k_pack_tc_f32(const float *__restrict__ data, float *__restrict__ out, int64_t nnzb, int R, int C) {
+    const int64_t total = nnzb * R * C;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = e / ((int64_t)R * C);
+        const int rc = (int)(e - p * R * C);
+        const int n = rc / C, k = rc - n * C;
+        const int64_t at = p * R * C * 2 + (k >> 3) * (R * 8) + (n >> 3) * 64 + ((k & 7) >> 2) * 32 + (n & 7) * 4 + (k & 3);
+        const float w = data[e];
+        const float h = __uint_as_float(__float_as_uint(w) & 0xffffe000u);
+        out[at] = h;
+        out[at + (int64_t)R * C] = w - h;
+    }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
@@ -371,8 +475,9 @@ uint32_t tmem_cols_for(int cols) {
     return n;
 }
 
-template <int R>
+template <typename T, int R>
 cudaError_t launch_r(const LaunchArgs &la, int G) {
+    constexpr int NS = TcCfg<T>::NS, KC = TcCfg<T>::KC;
     const Schedule &sc = *la.sc;
     const int n_items = (int)sc.items.size();
     if (n_items == 0 || la.N == 0) return cudaSuccess;
@@ -386,9 +491,9 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.n_tasks = (n_items + G - 1) / G;
     a.trec = sc.tc.d_rec[gidx];
     a.trec_off = sc.tc.d_rec_off[gidx];
-    a.wpk = static_cast<const uint16_t *>(la.data);
+    a.wpk = la.data;
     a.bias = la.bias;
-    a.Y = static_cast<uint16_t *>(la.Y);
+    a.Y = la.Y;
     a.ws = la.ws;
     a.status = la.status;
     a.N = la.N;
@@ -396,11 +501,11 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.M = sc.M;
     a.C = sc.C;
     a.nchunks = (int)((sc.K + KC - 1) / KC);
-    a.w_off = NS * kStageBytes;
+    a.w_off = (sizeof(T) == 4 ? 2 : 1) * NS * kStageBytes;
     a.trec_smem = a.w_off + (uint32_t)((sc.tc.task_wbytes[gidx] + 15) & ~size_t(15));
     a.bias_off = a.trec_smem + (uint32_t)((sc.tc.task_ibytes[gidx] + 15) & ~size_t(15));
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * R * 4 + 15) & ~size_t(15));
-    a.misc_off = a.bar_off + (2 * NS + 3) * 8;
+    a.misc_off = a.bar_off + (3 * NS + 3) * 8;
     a.tmem_cols = tmem_cols_for(G * R);
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
@@ -411,23 +516,24 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     cudaGetDevice(&dev);
     const uint64_t bit = 1ull << (dev & 63);
     if (!(attr_set.load() & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(k_tc<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem);
+        cudaError_t e = cudaFuncSetAttribute(k_tc<T, R>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem);
         if (e != cudaSuccess) return e;
         attr_set.fetch_or(bit);
     }
     CUtensorMap map;
     const cuuint64_t dims[2] = {(cuuint64_t)sc.K, (cuuint64_t)la.N};
-    const cuuint64_t strides[1] = {(cuuint64_t)sc.K * 2};
+    const cuuint64_t strides[1] = {(cuuint64_t)sc.K * sizeof(T)};
     const cuuint32_t box[2] = {(cuuint32_t)KC, (cuuint32_t)TN};
     const cuuint32_t estr[2] = {1, 1};
-    if (enc(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(la.X), dims, strides, box, estr,
+    if (enc(&map, sizeof(T) == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+            const_cast<void *>(la.X), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return cudaErrorInvalidValue;
     const int64_t n_tiles = (la.N + TN - 1) / TN;
     const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
     if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-    k_tc<R><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
+    k_tc<T, R><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
     return cudaGetLastError();
 }
 
@@ -435,8 +541,12 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
 
 bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
     const bool r_ok = R == 16 || R == 32 || R == 64 || R == 128;
-    const bool c_ok = C == 16 || C == 32 || C == 64;
-    return dt == BSR_BF16 && r_ok && c_ok && K % 8 == 0 && K > 0;
+    if (dt == BSR_BF16) return r_ok && (C == 16 || C == 32 || C == 64) && K % 8 == 0 && K > 0;
+    // fp32 as 3xTF32; a block lies inside one 32-column stage. Only blocks of
+    // 32 or more rows: each split stage then feeds enough MMA work; for 16-row
+    // blocks the SIMT kernel measured faster (the split adds a step to every
+    // stage's round trip)
+    return (R >= 32 && r_ok) && (C == 16 || C == 32) && K % 4 == 0 && K > 0;
 }
 
 int tc_g_index(int G) {
@@ -445,34 +555,44 @@ int tc_g_index(int G) {
     return 0;
 }
 
-size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes) {
-    return (size_t)NS * kStageBytes + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (2 * NS + 3) * 8 + (4 + 6 * 32) * 4 + 1024;
+size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt) {
+    const size_t ring = dt == BSR_F32 ? (size_t)2 * kTcStagesF32 * kStageBytes : (size_t)kTcStages * kStageBytes;
+    const int ns = dt == BSR_F32 ? kTcStagesF32 : kTcStages;
+    return ring + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (3 * ns + 3) * 8 + (4 + 6 * 32) * 4 + 1024;
 }
 
-size_t tc_task_budget(int R) {
-    const size_t fixed = tc_smem_bytes(R, 32, 0, 0) + 64;
+size_t tc_task_budget(int R, bsr_dtype_t dt) {
+    const size_t fixed = tc_smem_bytes(R, 32, 0, 0, dt) + 64;
     return fixed >= (size_t)kTcMaxSmem ? 0 : (size_t)kTcMaxSmem - fixed;
 }
 
 uint32_t tc_block_offset(int kk) { return (uint32_t)kk * 2; }
 
-cudaError_t pack_tc_data(const void *data, int64_t nnzb, int R, int C, uint16_t *out, cudaStream_t s) {
+cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, void *out, cudaStream_t s) {
     const int64_t total = nnzb * R * C;
     if (total == 0) return cudaSuccess;
     const int grid = (int)std::min<int64_t>((total + 255) / 256, 1 << 20);
-    k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), out, nnzb, R, C);
+    if (dt == BSR_F32)
+        k_pack_tc_f32<<<grid, 256, 0, s>>>(static_cast<const float *>(data), static_cast<float *>(out), nnzb, R, C);
+    else
+        k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), static_cast<uint16_t *>(out), nnzb, R, C);
     return cudaGetLastError();
 }
 
-cudaError_t launch_tc(const LaunchArgs &la, int G) {
+template <typename T>
+cudaError_t launch_tc_t(const LaunchArgs &la, int G) {
     switch (la.sc->R) {
-        case 16: return launch_r<16>(la, G);
-        case 32: return launch_r<32>(la, G);
-        case 64: return launch_r<64>(la, G);
-        case 128: return launch_r<128>(la, G);
+        case 16: return launch_r<T, 16>(la, G);
+        case 32: return launch_r<T, 32>(la, G);
+        case 64: return launch_r<T, 64>(la, G);
+        case 128: return launch_r<T, 128>(la, G);
     }
     return cudaErrorNotSupported;
+}
+
+cudaError_t launch_tc(const LaunchArgs &la, int G) {
+    return la.sc->dt == BSR_F32 ? launch_tc_t<float>(la, G) : launch_tc_t<uint16_t>(la, G);
 }
 
 }  // namespace bsr

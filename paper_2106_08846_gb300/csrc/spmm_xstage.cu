@@ -160,6 +160,25 @@ struct Tile {
     }
 };
 
+#ifdef XS_PLAIN1
+// one output per lane: plain fp32 FMA, no operand pairs to form
+template <>
+struct Tile<1> {
+    float a[8];
+    __device__ __forceinline__ void zero() {
+#pragma unroll
+        for (int k = 0; k < 8; k++) a[k] = 0.f;
+    }
+    __device__ __forceinline__ void fma(const float (&x)[8], const f2_t (&wd)[1]) {
+        float w, w2;
+        unpack2(wd[0], w, w2);
+#pragma unroll
+        for (int i = 0; i < 8; i++) a[i] = fmaf(x[i], w, a[i]);
+    }
+    __device__ __forceinline__ float get(int i, int) const { return a[i]; }
+};
+#endif
+
 // The TR weights of one block column for this lane, each as a (w, w) pair.
 // With WD == 2 the packed values already hold every weight twice, so the
 // pairs come straight from shared loads.
@@ -225,17 +244,32 @@ __device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *s
         // group's columns fall in distinct banks), dealt round-robin to the
         // S warps of the item; lane group ks takes block ks of each group
         const int ngr = (hi - lo + NKS - 1) / NKS;
-#pragma unroll kUnroll
-        for (int jg = piece; jg < ngr; jg += S) {
-            const int lb = lo + jg * NKS + ks;
-            if (NKS > 1 && lb >= hi) continue;
-            const unsigned char *xp = st + ((uint32_t)idx[lb] ^ tgx);
-            float x[8];
-            f2_t wd[TR];
+        // U groups per step with every load issued before the first FMA:
+        // the loop is otherwise one dependent chain (record -> X -> FMA) per
+        // block, and a few warps per scheduler cannot hide it
+        constexpr int U = TR <= 2 ? 4 : 1;
+        for (int jg = piece; jg < ngr; jg += S * U) {
+            int lbu[U];
+            bool v[U];
+            uint32_t off[U];
 #pragma unroll
-            for (int i = 0; i < 8; i++) x[i] = ld_x(xp + i * 1024, T());
-            load_wd<TR>(wbase + lb * R * WD, wd);
-            acc.fma(x, wd);
+            for (int u = 0; u < U; u++) {
+                lbu[u] = lo + (jg + S * u) * NKS + ks;
+                v[u] = jg + S * u < ngr && lbu[u] < hi;
+                if (!v[u]) lbu[u] = lo;   // a valid position: loads stay in bounds, the FMA is skipped
+                off[u] = (uint32_t)idx[lbu[u]] ^ tgx;
+            }
+            float x[U][8];
+            f2_t wd[U][TR];
+#pragma unroll
+            for (int u = 0; u < U; u++) {
+#pragma unroll
+                for (int i = 0; i < 8; i++) x[u][i] = ld_x(st + off[u] + i * 1024, T());
+                load_wd<TR>(wbase + lbu[u] * R * WD, wd[u]);
+            }
+#pragma unroll
+            for (int u = 0; u < U; u++)
+                if (v[u]) acc.fma(x[u], wd[u]);
         }
         return;
     } else {

@@ -270,7 +270,8 @@ def test_error_statuses():
     assert h.check_device_status() == b.BSR_OK
 
 
-@pytest.mark.parametrize("R,C,dtype,variant", [(32, 1, "f32", "xstage"), (16, 16, "bf16", "tcgen05")])
+@pytest.mark.parametrize("R,C,dtype,variant", [(32, 1, "f32", "xstage"), (16, 16, "bf16", "tcgen05"),
+                                               (32, 32, "f32", "tcgen05")])
 def test_bounded_wait_times_out_and_reports(monkeypatch, R, C, dtype, variant):
     """An X chunk that is never loaded: every wait on it gives up after the
     bound (2 ms here), the kernel records BSR_ERR_TIMEOUT, releases what it
@@ -303,3 +304,27 @@ def test_tensor_core_path_is_used_for_bf16_square_blocks(R, C):
     h, _, Y = _run(w, X)
     assert h.schedule()["variant"] == "tcgen05"
     check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, 256)
+
+
+@pytest.mark.parametrize("R,C", [(32, 32), (32, 16), (64, 16), (64, 32)])
+def test_tensor_core_path_is_used_for_fp32_square_blocks(R, C):
+    """fp32 blocks with both sides multiples of 16 run on the tensor cores as
+    three tf32 products (high x high + high x low + low x high) and must meet
+    the fp32 tolerance."""
+    w = _weight(256, 512, R, C, "f32", 0.25, 40 + R + C)
+    X = synth.activations(41, 200, 512, "f32")
+    h, _, Y = _run(w, X)
+    assert h.schedule()["variant"] == "tcgen05"
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, 256)
+
+
+def test_fp32_tensor_core_path_handles_large_magnitudes_and_tails():
+    """3xTF32 keeps fp32 accuracy across magnitudes: inputs scaled over a wide
+    range, a ragged token tail and K not a multiple of the 32-column stage."""
+    R, C = 32, 16
+    w = _weight(128, 16 * 21, R, C, "f32", 0.4, 77)
+    X = synth.activations(78, 131, 16 * 21, "f32") * np.float32(3.0e3)
+    X[::7] *= np.float32(1e-3)
+    h, _, Y = _run(w, X)
+    assert h.schedule()["variant"] == "tcgen05"
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, w.M)
