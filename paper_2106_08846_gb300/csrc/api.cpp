@@ -381,7 +381,8 @@ bsr_status_t bsr_check_device_status(bsr_handle_t h) {
 bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
     if (!h || !buf || len == 0) return BSR_ERR_INVALID_ARG;
     const Schedule &sc = *h->sched;
-    int64_t split_rows = (int64_t)sc.splits.size();
+    int64_t split_rows = 0;   // rows split into pieces (the other reduce entries are empty rows)
+    for (const Split &sp : sc.splits) split_rows += sp.nslot > 0;
     snprintf(buf, len,
              "variant=%s\ndtype=%s\nR=%d\nC=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
              "\nKB=%" PRId64 "\nnnzb=%" PRId64 "\ntokens_per_cta=%d\nthreads=%d\nsmem_bytes=%zu\n"

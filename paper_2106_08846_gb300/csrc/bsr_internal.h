@@ -23,7 +23,8 @@ struct Item {
     int32_t row, p0, p1, slot;
 };
 
-// A block row split into pieces: slots [slot0, slot0 + nslot) in piece order.
+// A row finished by the reduce pass: a block row split into pieces, slots
+// [slot0, slot0 + nslot) in piece order, or an empty row (nslot 0: Y = bias).
 struct Split {
     int32_t row, slot0, nslot, pad;
 };

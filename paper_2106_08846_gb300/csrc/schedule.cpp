@@ -31,8 +31,10 @@ cudaError_t upload(T **dst, const std::vector<T> &v) {
 }
 
 // Splits rows longer than `limit` blocks into ceil(len/limit) near-equal
-// pieces; orders the items longest first (LPT).
-void make_items(Schedule &sc, int64_t limit) {
+// pieces; orders the items longest first (LPT). With `drop_empty`, rows
+// without blocks get no item: the reduce pass writes their bias (a split
+// with no slots), so no CTA streams X for them.
+void make_items(Schedule &sc, int64_t limit, bool drop_empty = false) {
     sc.items.clear();
     sc.splits.clear();
     sc.n_slots = 0;
@@ -40,6 +42,10 @@ void make_items(Schedule &sc, int64_t limit) {
     for (int64_t i = 0; i < sc.MB; i++) {
         int32_t p0 = sc.indptr[i], p1 = sc.indptr[i + 1];
         int64_t len = p1 - p0;
+        if (drop_empty && len == 0) {
+            sc.splits.push_back({(int32_t)i, 0, 0, 0});
+            continue;
+        }
         if (limit <= 0 || len <= limit) {
             sc.items.push_back({(int32_t)i, p0, p1, -1});
             continue;
@@ -307,7 +313,7 @@ bsr_status_t build_schedule(Schedule &sc) {
         const int64_t lmax = std::max<int64_t>(1, avail / (int64_t)(tc_block_bytes(sc.R, sc.C, sc.dt) + 4));
         int64_t limit = split_limit(sc);
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
-        make_items(sc, limit);
+        make_items(sc, limit, true);
         plan_tc(sc);
     } else if (!want_generic && xstage_supports(sc.R, sc.C, sc.dt, sc.K)) {
         sc.variant = V_XSTAGE;
@@ -320,7 +326,7 @@ bsr_status_t build_schedule(Schedule &sc) {
             std::max<int64_t>(1, avail / (int64_t)((size_t)sc.R * sc.C * 4 * kXsWDup + 4));
         int64_t limit = split_limit(sc);
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
-        make_items(sc, limit);
+        make_items(sc, limit, sc.R > 1);   // one-row blocks keep their rare empty rows: tasks stay row-contiguous
         plan_xstage(sc);
     }
     if (sc.variant == V_XSTAGE && (int64_t)sc.xs_blob.size() > INT32_MAX) sc.variant = V_GENERIC;   // blob offsets are int32
