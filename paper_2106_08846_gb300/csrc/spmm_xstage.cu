@@ -56,7 +56,6 @@ constexpr int TN = kXsTokens;
 constexpr int KC = kXsChunk;
 constexpr int NS = kXsStages;
 constexpr int NCW = kXsConsumerWarps;
-constexpr int NTHREADS = (NCW + 1) * 32;
 constexpr int WD = kXsWDup;
 constexpr int kItab = kXsItab;   // ints per item in a task's item table
 #ifndef XS_UNROLL
@@ -160,8 +159,8 @@ struct Tile {
     }
 };
 
-#ifdef XS_PLAIN1
-// one output per lane: plain fp32 FMA, no operand pairs to form
+// one output per lane: plain fp32 FMA, no operand pairs to form (measured
+// faster than the packed form for this load-bound tile)
 template <>
 struct Tile<1> {
     float a[8];
@@ -177,7 +176,6 @@ struct Tile<1> {
     }
     __device__ __forceinline__ float get(int i, int) const { return a[i]; }
 };
-#endif
 
 // The TR weights of one block column for this lane, each as a (w, w) pair.
 // With WD == 2 the packed values already hold every weight twice, so the
@@ -244,10 +242,9 @@ __device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *s
         // group's columns fall in distinct banks), dealt round-robin to the
         // S warps of the item; lane group ks takes block ks of each group
         const int ngr = (hi - lo + NKS - 1) / NKS;
-        // U groups per step with every load issued before the first FMA:
-        // the loop is otherwise one dependent chain (record -> X -> FMA) per
-        // block, and a few warps per scheduler cannot hide it
-        constexpr int U = TR <= 2 ? 4 : 1;
+        // (U groups per step with all loads first measured no faster: the
+        // shared-memory pipe, not one warp's dependent chain, sets the pace)
+        constexpr int U = 1;
         for (int jg = piece; jg < ngr; jg += S * U) {
             int lbu[U];
             bool v[U];
@@ -380,31 +377,31 @@ __device__ __forceinline__ void store_tile(const XsArgs &a, const Shared &sh, co
     }
 }
 
-// Consumer warps. RW == 1: S = 12/G warps share each item (block-strided)
-// and a pairwise tree sums them. RW > 1 (G = 12 RW): each warp owns RW
+// NW consumer warps. RW == 1: S = NW/G warps share each item (block-strided)
+// and a pairwise tree sums them. RW > 1 (G = NW RW): each warp owns RW
 // whole items, with one register tile each, and needs no tree.
-template <typename T, int TR, int NRG, int CT, int RW>
+template <typename T, int TR, int NRG, int CT, int RW, int NW>
 __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int64_t n0, int task,
                                          int g_count, uint32_t CL, int warp, int lane) {
     using St = Stage<T>;
     constexpr int R = TR * NRG;
     const int C = CT ? CT : a.C;
     const int nch = a.nchunks;
-    const int ctid = threadIdx.x;   // 0 .. NCW*32-1
+    const int ctid = threadIdx.x;   // 0 .. NW*32-1
 
     // ---- the task's blob (item table, records, block values) in one round
     // trip: 16-byte asynchronous copies from all consumer threads
     if (g_count > 0) {
         const int4 *src = reinterpret_cast<const int4 *>(a.blob + (int64_t)task * a.stride);
         int4 *dst = reinterpret_cast<int4 *>(sh.itab);
-        for (int e = ctid; e < (int)(a.stride / 16); e += NCW * 32) ptx::cp_async16(dst + e, src + e);
+        for (int e = ctid; e < (int)(a.stride / 16); e += NW * 32) ptx::cp_async16(dst + e, src + e);
     }
     ptx::cp_async_wait_all();
-    ptx::named_barrier(1, NCW * 32);
+    ptx::named_barrier(1, NW * 32);
     // the bias, needed only by the epilogue (waited for there), and whether
     // the task covers consecutive whole rows (then the epilogue stores whole
     // row segments of Y)
-    for (int e = ctid; e < g_count * R; e += NCW * 32) {
+    for (int e = ctid; e < g_count * R; e += NW * 32) {
         const int g = e / R, r = e - g * R;
         if (a.bias)
             ptx::cp_async4(&sh.B[e], a.bias + (int64_t)sh.itab[kItab * g + 0] * R + r);
@@ -451,7 +448,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
             atomicExch(&sh.misc[0], 1);
         }
         ptx::cp_async_wait_all();   // the bias
-        if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
+        if (ptx::named_barrier_or(1, NW * 32, !ok || aborted(sh.misc))) return;
         if (R == 1 && sh.misc[3]) {
             // consecutive rows row0 .. row0+G-1: transpose the tiles through
             // shared memory (the ring is free) and store Y row segments
@@ -466,9 +463,9 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
 #pragma unroll
                     for (int i = 0; i < 8; i++) P[(tg + 8 * i) * PG + gi] = v[i][0];
             }
-            ptx::named_barrier(1, NCW * 32);
+            ptx::named_barrier(1, NW * 32);
             const int64_t row0 = sh.itab[0];
-            for (int e = ctid; e < TN * g_count; e += NCW * 32) {
+            for (int e = ctid; e < TN * g_count; e += NW * 32) {
                 const int t = e / g_count, j = e - t * g_count;
                 const int64_t n = n0 + t;
                 if (n < a.N)
@@ -519,7 +516,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     // every consumer is done with the ring and the block values; the abort
     // verdict is the same for all of them (barrier reduction)
     ptx::cp_async_wait_all();   // the bias
-    if (ptx::named_barrier_or(1, NCW * 32, !ok || aborted(sh.misc))) return;
+    if (ptx::named_barrier_or(1, NW * 32, !ok || aborted(sh.misc))) return;
     // pairwise tree over the S warps of each item: in round `step`, the warp
     // of piece p (p % 2step == step) hands its tile to piece p - step
     constexpr int PS = R + 4;          // padded row of a tile in shared memory (16-byte aligned)
@@ -541,7 +538,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
                 }
             }
         }
-        ptx::named_barrier(1, NCW * 32);
+        ptx::named_barrier(1, NW * 32);
         if (has_item && piece % (2 * step) == 0 && piece + step < S) {
 #pragma unroll
             for (int i = 0; i < 8; i++) {
@@ -561,14 +558,14 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
                 }
             }
         }
-        ptx::named_barrier(1, NCW * 32);
+        ptx::named_barrier(1, NW * 32);
     }
     if (!has_item || piece != 0 || ks != 0) return;
     store_tile<T, TR, NRG>(a, sh, v, gi, n0, rg, tg);
 }
 
-template <typename T, int TR, int NRG, int CT, int RW>
-__global__ void __launch_bounds__(NTHREADS, 1)
+template <typename T, int TR, int NRG, int CT, int RW, int NW>
+__global__ void __launch_bounds__((NW + 1) * 32, 1)
 k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     using St = Stage<T>;
     constexpr int R = TR * NRG;
@@ -599,7 +596,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; s++) {
             ptx::mbar_init(&sh.full[s], 1);
-            ptx::mbar_init(&sh.empty[s], NCW * CL);
+            ptx::mbar_init(&sh.empty[s], NW * CL);
         }
         sh.misc[0] = 0;
         sh.misc[3] = 1;
@@ -608,7 +605,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     // every CTA's barriers exist before any multicast or remote arrive
     if (CL == 1) __syncthreads(); else ptx::cluster_sync();
 
-    if (warp == NCW) {
+    if (warp == NW) {
         // ---------------- producer: block values by bulk copy, then X chunks
         if (lane == 0) {
             ptx::prefetch_tensormap(&xmap);
@@ -643,7 +640,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
         }
         __syncwarp();
     } else {
-        consumer<T, TR, NRG, CT, RW>(a, sh, n0, task, g_count, CL, warp, lane);
+        consumer<T, TR, NRG, CT, RW, NW>(a, sh, n0, task, g_count, CL, warp, lane);
     }
     if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
 }
@@ -691,13 +688,14 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // ring, reused for the epilogue's partial tiles
 size_t region_bytes(bsr_dtype_t dt, int R) {
     const size_t ring = (size_t)NS * (dt == BSR_F32 ? Stage<float>::kBytes : Stage<uint16_t>::kBytes);
-    const size_t part = (size_t)(NCW * 2 / 3) * TN * (R + 4) * 4;   // most tiles of one tree round (G=4, S=3)
+    const int nw = R == 1 ? kXsConsumerWarpsR1 : NCW;
+    const size_t part = (size_t)(nw * 2 / 3) * TN * (R + 4) * 4;   // most tiles of one tree round (S=3)
     return (std::max(ring, part) + 1023) & ~size_t(1023);
 }
 
 // Whether clusters of CL CTAs with `smem` bytes each can be resident at all
 // (cached per kernel, cluster size, shared-memory size and device).
-bool cluster_fits(const void *func, int CL, uint32_t smem, int dev) {
+bool cluster_fits(const void *func, int CL, uint32_t smem, int dev, int threads) {
     struct Entry {
         const void *func;
         int CL, dev;
@@ -711,7 +709,7 @@ bool cluster_fits(const void *func, int CL, uint32_t smem, int dev) {
         if (e.func == func && e.CL == CL && e.smem == smem && e.dev == dev) return e.ok;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)CL);
-    cfg.blockDim = dim3(NTHREADS);
+    cfg.blockDim = dim3((unsigned)threads);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -738,7 +736,7 @@ int choose_cluster(int n_tasks) {
     return 1;
 }
 
-template <typename T, int TR, int NRG, int CT, int RW>
+template <typename T, int TR, int NRG, int CT, int RW, int NW>
 cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     const Schedule &sc = *la.sc;
     const size_t es = sizeof(T);
@@ -752,7 +750,8 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     XsArgs a;
     a.n_items = n_items;
     a.G = G;
-    a.S = G <= NCW ? NCW / G : 1;
+    a.S = G <= NW ? NW / G : 1;
+    constexpr int NTHREADS = (NW + 1) * 32;
     a.n_tasks = (n_items + G - 1) / G;
     a.blob = static_cast<const unsigned char *>(la.data) + sc.xs_blob_off[gidx];
     a.stride = (uint32_t)sc.xs_blob_stride[gidx];
@@ -779,7 +778,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     cudaGetDevice(&dev);
     const uint64_t bit = 1ull << (dev & 63);
     if (!(attr_set.load() & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG, CT, RW>,
+        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG, CT, RW, NW>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kXsMaxSmem);
         if (e != cudaSuccess) return e;
         attr_set.fetch_or(bit);
@@ -789,7 +788,8 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
 
     cudaError_t err = cudaErrorInvalidConfiguration;
     for (int CL = choose_cluster(a.n_tasks); CL >= 1; CL >>= 1) {
-        if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT, RW>), CL, smem, dev))
+        if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT, RW, NW>), CL, smem, dev,
+                                    NTHREADS))
             continue;
         const int64_t n_groups = (a.n_tasks + CL - 1) / CL;
         const int64_t grid = n_tiles * n_groups * CL;   // cluster-major, tile-fastest
@@ -805,7 +805,7 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
         if (CL == 1) {
-            k_xstage<T, TR, NRG, CT, RW><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
+            k_xstage<T, TR, NRG, CT, RW, NW><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
             err = cudaGetLastError();
             break;
         }
@@ -821,23 +821,29 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
         attr[0].val.clusterDim.z = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        err = cudaLaunchKernelEx(&cfg, k_xstage<T, TR, NRG, CT, RW>, map, a);
+        err = cudaLaunchKernelEx(&cfg, k_xstage<T, TR, NRG, CT, RW, NW>, map, a);
         break;
     }
     return err;
 }
 
-// Items per consumer warp: G = 12 RW with RW > 1 only for one-row blocks.
+// One-row blocks: kXsConsumerWarpsR1 consumer warps (their register tiles
+// are small, and more warps hide the shared-memory latency of the one-load-
+// per-FMA loop), each owning G/NW items when G exceeds them. Other blocks:
+// kXsConsumerWarps, G <= NW.
 template <typename T, int TR, int NRG, int CT>
 cudaError_t launch_w(const LaunchArgs &la, const XsPlan &pl, int G) {
     if constexpr (TR == 1 && NRG == 1) {
-        switch (G / NCW) {
-            case 2: return launch_t<T, TR, NRG, CT, 2>(la, pl, G);
-            case 4: return launch_t<T, TR, NRG, CT, 4>(la, pl, G);
+        constexpr int NW = kXsConsumerWarpsR1;
+        switch (G > NW ? G / NW : 1) {
+            case 1: return G <= NW ? launch_t<T, TR, NRG, CT, 1, NW>(la, pl, G) : cudaErrorInvalidConfiguration;
+            case 2: return launch_t<T, TR, NRG, CT, 2, NW>(la, pl, G);
         }
+        return cudaErrorInvalidConfiguration;
+    } else {
+        if (G > NCW) return cudaErrorInvalidConfiguration;
+        return launch_t<T, TR, NRG, CT, 1, NCW>(la, pl, G);
     }
-    if (G > NCW) return cudaErrorInvalidConfiguration;
-    return launch_t<T, TR, NRG, CT, 1>(la, pl, G);
 }
 
 template <typename T, int TR, int NRG>
@@ -882,7 +888,10 @@ int g_index(int G) {
     return 0;
 }
 
-bool xstage_task_size_ok(int R, int G) { return G <= kXsConsumerWarps || R == 1; }
+bool xstage_task_size_ok(int R, int G) {
+    return R == 1 ? (G <= kXsConsumerWarpsR1 ? kXsConsumerWarpsR1 % G == 0 : G == 2 * kXsConsumerWarpsR1)
+                  : G <= kXsConsumerWarps;
+}
 
 bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
     const bool r_ok = R == 1 || R == 2 || R == 4 || R == 8 || R == 16 || R == 32;

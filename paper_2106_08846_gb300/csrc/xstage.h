@@ -12,12 +12,13 @@ constexpr int kXsTokens = 64;          // tokens per CTA
 constexpr int kXsChunk = 128;          // K columns per ring stage
 constexpr int kXsStages = 3;           // ring depth
 constexpr int kXsConsumerWarps = 12;   // + 1 producer warp: 16 warps of registers
+constexpr int kXsConsumerWarpsR1 = 24; // one-row blocks (small tiles): + 1 producer warp, 80 registers a thread
 constexpr int kXsMaxSmem = 232448;     // 227 KB, the per-CTA opt-in limit
 constexpr int kXsWDup = 1;             // copies of each packed block value
 
-// Task sizes G (items per CTA): up to 12, each divides the consumer warps
-// (12/G warps per item); above 12, each warp owns G/12 items (one-row
-// blocks only, whose register tiles are small).
+// Task sizes G (items per CTA): up to the consumer warps NW, each dividing
+// them (NW/G warps per item); one-row blocks (NW = 24) also G = 48, two
+// items per warp.
 constexpr int kXsTaskSizes = 8;
 constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12, 24, 48};
 
