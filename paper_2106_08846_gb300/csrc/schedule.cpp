@@ -135,6 +135,7 @@ void quad_order(Schedule &sc, int32_t p0, int32_t lo, int32_t hi) {
 template <typename F>
 void build_records(Schedule &sc, int chunk, F value) {
     const int64_t nch = (sc.K + chunk - 1) / chunk;
+    const int bi = xstage_block_ints(sc.R, sc.C);
     sc.xs_rec.clear();
     sc.xs_rec_off.assign(sc.items.size(), 0);
     sc.xs_perm.assign((size_t)sc.nnzb, 0);
@@ -143,9 +144,9 @@ void build_records(Schedule &sc, int chunk, F value) {
         const int32_t len = it.p1 - it.p0;
         sc.xs_rec_off[i] = (int32_t)sc.xs_rec.size();
         const size_t base = sc.xs_rec.size();
-        sc.xs_rec.resize(base + (size_t)xstage_record_ints(len, nch), 0);
+        sc.xs_rec.resize(base + (size_t)xstage_record_ints(len, nch, bi), 0);
         int32_t b = 0;
-        const size_t cbase = base + (size_t)xstage_pad4(len);
+        const size_t cbase = base + (size_t)xstage_pad4(bi * len);
         for (int64_t c = 0; c <= nch; c++) {
             const int64_t first_col = c * (chunk / sc.C);
             while (b < len && sc.indices[it.p0 + b] < first_col) b++;
@@ -156,8 +157,8 @@ void build_records(Schedule &sc, int chunk, F value) {
         if (sc.C == 1)
             for (int64_t c = 0; c < nch; c++)
                 quad_order(sc, it.p0, sc.xs_rec[cbase + c], sc.xs_rec[cbase + c + 1]);
-        for (int32_t k = 0; k < len; k++)
-            sc.xs_rec[base + k] = value((int64_t)sc.indices[sc.xs_perm[(size_t)it.p0 + k]]);
+        for (int32_t k = 0; k < len; k++)   // (a 1x1 block's weight slot is filled by the value packing)
+            sc.xs_rec[base + (size_t)bi * k] = value((int64_t)sc.indices[sc.xs_perm[(size_t)it.p0 + k]]);
     }
 }
 
@@ -175,7 +176,7 @@ void footprints(const Schedule &sc, size_t per_block, int chunk, const int *Gs, 
             for (size_t k = t; k < std::min(sc.items.size(), t + G); k++) {
                 const int64_t len = sc.items[k].p1 - sc.items[k].p0;
                 blocks += (size_t)xstage_pad4(len * (int64_t)per_block / 4) * 4;
-                rec += (size_t)xstage_record_ints(len, nch) * 4;
+                rec += (size_t)xstage_record_ints(len, nch, xstage_block_ints(sc.R, sc.C)) * 4;
             }
             wmax = std::max(wmax, blocks);
             imax = std::max(imax, rec);
@@ -189,7 +190,8 @@ void plan_xstage(Schedule &sc) {
     build_records(sc, kXsChunk, [&](int64_t col) {
         return sc.C == 1 ? (int32_t)xstage_stage_offset(sc.dt, (int)(col % kXsChunk)) : (int32_t)col;
     });
-    const int per_block = sc.R * sc.C * kXsWDup;   // floats
+    const int bi = xstage_block_ints(sc.R, sc.C);
+    const int per_block = bi == 2 ? 0 : sc.R * sc.C * kXsWDup;   // floats in the value region (1x1: in the records)
     footprints(sc, (size_t)per_block * 4, kXsChunk, kXsG, kXsTaskSizes, sc.xs.task_wbytes, sc.xs.task_ibytes);
     // the task blobs of every task size that fits: layout, then the template
     const int64_t n = (int64_t)sc.items.size();
@@ -219,7 +221,7 @@ void plan_xstage(Schedule &sc) {
             for (int64_t k = 0; k < G && t * G + k < n; k++) {
                 const int64_t i = t * G + k;
                 const Item &it = sc.items[(size_t)i];
-                const int64_t len = it.p1 - it.p0, rints = xstage_record_ints(len, nch);
+                const int64_t len = it.p1 - it.p0, rints = xstage_record_ints(len, nch, bi);
                 int32_t *h = &sc.xs_blob[(size_t)(blob + k * kXsItab)];
                 h[0] = it.row;
                 h[1] = it.p0;
@@ -230,7 +232,7 @@ void plan_xstage(Schedule &sc) {
                 h[8] = (int32_t)roff;
                 std::copy(sc.xs_rec.begin() + sc.xs_rec_off[(size_t)i], sc.xs_rec.begin() + sc.xs_rec_off[(size_t)i] + rints,
                           sc.xs_blob.begin() + (recs + roff));
-                if (len) sc.xs_vdst[(size_t)(gi * n + i)] = vals + woff;
+                if (len) sc.xs_vdst[(size_t)(gi * n + i)] = bi == 2 ? recs + roff + 1 : vals + woff;
                 woff += xstage_pad4(len * per_block);
                 roff += rints;
             }

@@ -254,15 +254,22 @@ __device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *s
                 lbu[u] = lo + (jg + S * u) * NKS + ks;
                 v[u] = jg + S * u < ngr && lbu[u] < hi;
                 if (!v[u]) lbu[u] = lo;   // a valid position: loads stay in bounds, the FMA is skipped
-                off[u] = (uint32_t)idx[lbu[u]] ^ tgx;
             }
             float x[U][8];
             f2_t wd[U][TR];
 #pragma unroll
             for (int u = 0; u < U; u++) {
+                if constexpr (R == 1) {
+                    // 1x1: (X offset, weight) in one 8-byte record entry
+                    const int2 ow = reinterpret_cast<const int2 *>(idx)[lbu[u]];
+                    off[u] = (uint32_t)ow.x ^ tgx;
+                    wd[u][0] = pack2(__int_as_float(ow.y), __int_as_float(ow.y));
+                } else {
+                    off[u] = (uint32_t)idx[lbu[u]] ^ tgx;
+                    load_wd<TR>(wbase + lbu[u] * R * WD, wd[u]);
+                }
 #pragma unroll
                 for (int i = 0; i < 8; i++) x[u][i] = ld_x(st + off[u] + i * 1024, T());
-                load_wd<TR>(wbase + lbu[u] * R * WD, wd[u]);
             }
 #pragma unroll
             for (int u = 0; u < U; u++)
@@ -388,6 +395,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     const int C = CT ? CT : a.C;
     const int nch = a.nchunks;
     const int ctid = threadIdx.x;   // 0 .. NW*32-1
+    const int BI = xstage_block_ints(R, C);   // record ints per block
 
     // ---- the task's blob (item table, records, block values) in one round
     // trip: 16-byte asynchronous copies from all consumer threads
@@ -431,7 +439,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
                 const int gi = warp * RW + r;
                 if (gi < g_count) {
                     const int32_t *idx = sh.I + sh.itab[kItab * gi + 8];
-                    const int32_t *cb = idx + xstage_pad4(sh.itab[kItab * gi + 5]);
+                    const int32_t *cb = idx + xstage_pad4(BI * sh.itab[kItab * gi + 5]);
                     const float *wbase = sh.W + sh.itab[kItab * gi + 7] + rg * TR * WD;
                     item_chunk<T, TR, NRG, CT>(acc[r], st, idx, cb, wbase, c, 0, 1, ks, tgx, C);
                 }
@@ -487,7 +495,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     const int gi = warp / S, piece = warp % S;
     const bool has_item = gi < g_count;
     const int32_t *idx = sh.I + (has_item ? sh.itab[kItab * gi + 8] : 0);
-    const int32_t *cb = idx + (has_item ? xstage_pad4(sh.itab[kItab * gi + 5]) : 0);
+    const int32_t *cb = idx + (has_item ? xstage_pad4(BI * sh.itab[kItab * gi + 5]) : 0);
     const float *wbase = sh.W + (has_item ? sh.itab[kItab * gi + 7] : 0) + rg * TR * WD;
 
     Tile<TR> acc;
@@ -648,10 +656,12 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
 // Block values into the task blobs of every task size: item i's values go to
 // blobs + vdst[g * n_items + i] (floats; -1: none), blocks in the records'
 // order (perm: position -> stored block), per block W^T widened to fp32
-// with WD copies: [(b*C + c)*R + r]*WD + d <- data[(perm[p0_i + b]*R + r)*C + c].
+// with WD copies: [(b*C + c)*R + r]*stride + d <- data[(perm[p0_i + b]*R + r)*C + c]
+// (stride WD, or 2 for 1x1 blocks whose weights sit beside their offsets).
 template <typename T>
 __global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ items, const int32_t *__restrict__ perm,
-                       const int64_t *__restrict__ vdst, int64_t n_items, float *__restrict__ blobs, int R, int C) {
+                       const int64_t *__restrict__ vdst, int64_t n_items, float *__restrict__ blobs, int R, int C,
+                       int stride) {
     for (int64_t gi = blockIdx.x; gi < kXsTaskSizes * n_items; gi += gridDim.x) {
         const int64_t d = vdst[gi];
         if (d < 0) continue;
@@ -663,8 +673,7 @@ __global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ item
             const int rc = (int)(e - b * R * C);
             const int c = rc / R, r = rc - c * R;
             const float w = to_f32(data[((int64_t)perm[it.p0 + b] * R + r) * C + c]);
-#pragma unroll
-            for (int k = 0; k < WD; k++) dst[WD * e + k] = w;
+            for (int k = 0; k < WD; k++) dst[stride * e + k] = w;
         }
     }
 }
@@ -904,10 +913,11 @@ cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items
                              const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s) {
     if (n_items == 0) return cudaSuccess;
     const int grid = (int)std::min<int64_t>(kXsTaskSizes * n_items, 1 << 16);
+    const int stride = xstage_block_ints(R, C) == 2 ? 2 : WD;
     if (dt == BSR_F32)
-        k_pack<float><<<grid, 256, 0, s>>>((const float *)data, items, perm, vdst, n_items, blobs, R, C);
+        k_pack<float><<<grid, 256, 0, s>>>((const float *)data, items, perm, vdst, n_items, blobs, R, C, stride);
     else
-        k_pack<uint16_t><<<grid, 256, 0, s>>>((const uint16_t *)data, items, perm, vdst, n_items, blobs, R, C);
+        k_pack<uint16_t><<<grid, 256, 0, s>>>((const uint16_t *)data, items, perm, vdst, n_items, blobs, R, C, stride);
     return cudaGetLastError();
 }
 

@@ -38,18 +38,23 @@ struct XsPlan {
     size_t task_ibytes[kXsTaskSizes] = {};   // item records (see xstage_record_ints)
 };
 
-// Per item, the kernel fetches one "record" of int32 by bulk copy:
+// Per item, the task blob holds one "record" of int32:
 //   [ per block: its X offset inside a ring stage (C == 1) or its block
-//     column (C > 1), padded to 4 ints | per K chunk c = 0..nchunks: the
-//     first item-local block of chunk c, padded to 4 ints ]
+//     column (C > 1) -- for 1x1 blocks followed by its weight --, padded to
+//     4 ints | per K chunk c = 0..nchunks: the first item-local block of
+//     chunk c, padded to 4 ints ]
 #ifdef __CUDACC__
 #define XS_HD __host__ __device__
 #else
 #define XS_HD
 #endif
 XS_HD inline int64_t xstage_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
-XS_HD inline int64_t xstage_record_ints(int64_t len, int64_t nchunks) {
-    return xstage_pad4(len) + xstage_pad4(nchunks + 1);
+// ints per block in a record: 1x1 blocks carry (X offset, weight) pairs, so
+// one 8-byte load gives a block's whole operand description; others one int
+// (their values live in the blob's value region)
+XS_HD inline int xstage_block_ints(int R, int C) { return R == 1 && C == 1 ? 2 : 1; }
+XS_HD inline int64_t xstage_record_ints(int64_t len, int64_t nchunks, int bi = 1) {
+    return xstage_pad4(bi * len) + xstage_pad4(nchunks + 1);
 }
 // Byte offset of chunk column kk inside a ring stage, token row 0.
 uint32_t xstage_stage_offset(bsr_dtype_t dt, int kk);
