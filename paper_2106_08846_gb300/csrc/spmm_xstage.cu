@@ -15,12 +15,11 @@
 //    mbarrier counts the bytes of all slices; every consumer warp waits for
 //    every chunk in order, processes all of its blocks that fall in it, and
 //    releases the stage on the "empty" mbarrier of every CTA in the cluster.
-//  * Per task, the consumer threads copy in, with 16-byte cp.async (many
-//    in flight: one bulk copy per task streamed far slower), the block
-//    values (repacked at create time to fp32 [p][c][r], each item 16-byte
-//    aligned) and the items' records built on the host: each block's X
-//    offset inside a stage (1-column blocks) or block column, and the first
-//    block of every chunk, so the per-chunk loop has no search or test.
+//  * Per task, the producer bulk-copies one blob (built at create time):
+//    the item table, the items' records -- each block's X offset inside a
+//    stage (1-column blocks) or block column, and the first block of every
+//    chunk, so the per-chunk loop has no search or test -- and the block
+//    values (fp32 [p][c][r]; 1x1 weights sit in the records).
 //  * Lane = tg + 8 q: tg picks 8 tokens (tg, tg+8, ..., tg+56: conflict-free
 //    under the swizzle, which XORs the 16-byte column group with tg), q
 //    splits into NRG output groups of TR rows and NKS = 4/NRG lanes that take
@@ -219,7 +218,7 @@ __device__ __forceinline__ bool aborted(const int *flag) {
 
 struct Shared {
     unsigned char *base;
-    uint64_t *full, *empty;
+    uint64_t *full, *empty, *wbar;
     int *misc;          // [0] abort flag, [3] task covers consecutive whole rows
     int *itab;          // the blob's item table (kItab ints per item)
     float *W;           // block values of the task's items
@@ -397,14 +396,14 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     const int ctid = threadIdx.x;   // 0 .. NW*32-1
     const int BI = xstage_block_ints(R, C);   // record ints per block
 
-    // ---- the task's blob (item table, records, block values) in one round
-    // trip: 16-byte asynchronous copies from all consumer threads
-    if (g_count > 0) {
-        const int4 *src = reinterpret_cast<const int4 *>(a.blob + (int64_t)task * a.stride);
-        int4 *dst = reinterpret_cast<int4 *>(sh.itab);
-        for (int e = ctid; e < (int)(a.stride / 16); e += NW * 32) ptx::cp_async16(dst + e, src + e);
+    // ---- the task's blob (item table, records, block values): one bulk
+    // copy the producer issued first thing, one round trip
+    if (g_count > 0 && !__all_sync(0xffffffffu, ptx::mbar_wait_bounded(sh.wbar, 0, a.wait_ns))) {
+        if (lane == 0) {
+            set_status(a.status, DEV_TIMEOUT);
+            atomicExch(&sh.misc[0], 1);
+        }
     }
-    ptx::cp_async_wait_all();
     ptx::named_barrier(1, NW * 32);
     // the bias, needed only by the epilogue (waited for there), and whether
     // the task covers consecutive whole rows (then the epilogue stores whole
@@ -582,6 +581,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     sh.base = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     sh.full = reinterpret_cast<uint64_t *>(sh.base + a.bar_off);
     sh.empty = sh.full + NS;
+    sh.wbar = sh.empty + NS;
     sh.misc = reinterpret_cast<int *>(sh.base + a.misc_off);
     sh.itab = reinterpret_cast<int *>(sh.base + a.blob_off);
     sh.I = reinterpret_cast<int32_t *>(sh.base + a.blob_off + a.hdr);
@@ -606,6 +606,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
             ptx::mbar_init(&sh.full[s], 1);
             ptx::mbar_init(&sh.empty[s], NW * CL);
         }
+        ptx::mbar_init(sh.wbar, 1);
         sh.misc[0] = 0;
         sh.misc[3] = 1;
         ptx::fence_barrier_init();
@@ -616,6 +617,10 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     if (warp == NW) {
         // ---------------- producer: block values by bulk copy, then X chunks
         if (lane == 0) {
+            if (g_count > 0) {   // the task blob, then the X chunks
+                ptx::mbar_arrive_expect_tx(sh.wbar, a.stride);
+                ptx::bulk_load(sh.itab, a.blob + (int64_t)task * a.stride, a.stride, sh.wbar);
+            }
             ptx::prefetch_tensormap(&xmap);
             const int rows = TN / (int)CL;                       // this CTA's slice of every chunk
             const uint16_t mask = (uint16_t)((1u << CL) - 1u);
@@ -645,6 +650,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
             // them so that no TMA write outlives the CTA
             for (int d = max(0, c - NS); d < c; d++)
                 if (d != a.stall_chunk) ptx::mbar_wait_bounded(&sh.full[d % NS], (d / NS) & 1, kDrainNs);
+            if (g_count > 0) ptx::mbar_wait_bounded(sh.wbar, 0, kDrainNs);
         }
         __syncwarp();
     } else {
