@@ -134,8 +134,10 @@ bsr_status_t bsr_check_device_status(bsr_handle_t h);
 
 /*
  * bsr_get_schedule -- a text description of the handle's schedule: kernel
- * variant, tile sizes, work items, split rows, launches per call and the
- * schedule-cache statistics, as "key=value" lines. Writes at most len bytes
+ * variant, execution block width (exec_C: 64 where narrow bf16 blocks run on
+ * the tensor cores as zero-filled R x 64 tiles), tile sizes, work items, split
+ * rows, launches per call and the schedule-cache statistics, as "key=value"
+ * lines. Writes at most len bytes
  * including the terminating NUL into buf (truncating). Returns
  * BSR_ERR_INVALID_ARG for a NULL handle or buffer.
  */

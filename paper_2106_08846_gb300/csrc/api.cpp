@@ -118,6 +118,7 @@ Schedule::~Schedule() {
     cudaFree(d_group_begin);
     cudaFree(d_indptr);
     cudaFree(d_xs_perm);
+    cudaFree(d_vmap);
     cudaFree(d_xs_vdst);
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);
@@ -384,13 +385,13 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
     int64_t split_rows = 0;   // rows split into pieces (the other reduce entries are empty rows)
     for (const Split &sp : sc.splits) split_rows += sp.nslot > 0;
     snprintf(buf, len,
-             "variant=%s\ndtype=%s\nR=%d\nC=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
+             "variant=%s\ndtype=%s\nR=%d\nC=%d\nexec_C=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
              "\nKB=%" PRId64 "\nnnzb=%" PRId64 "\ntokens_per_cta=%d\nthreads=%d\nsmem_bytes=%zu\n"
              "item_groups=%d\nitems=%zu\nsplit_len=%d\nsplit_rows=%" PRId64 "\nslots=%d\n"
              "empty_rows=%" PRId64 "\nmax_row_blocks=%" PRId64 "\nlaunches_per_call=%d\n"
              "structure_hash=%016" PRIx64 "\ncache_hit=%d\nschedule_reuses=%" PRId64
              "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\n",
-             variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.M, sc.K,
+             variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_C, sc.M, sc.K,
              sc.MB, sc.KB, sc.nnzb, sc.tn, sc.threads, sc.smem, sc.groups, sc.items.size(),
              sc.split_len, split_rows, sc.n_slots, sc.empty_rows, sc.max_row, launches_per_call(sc),
              sc.hash, (int)h->cache_hit, (int64_t)sc.reuse_count, (int64_t)g_cache_hits,

@@ -80,6 +80,15 @@ struct Schedule {
     int32_t *d_indptr = nullptr;        // owned copies of the structure
     int32_t *d_indices = nullptr;
 
+    // Execution structure of the tensor-core kernel when it runs narrow bf16
+    // blocks re-blocked into R x 64 tiles (ex_C = 64; zeros for absent
+    // blocks): the items and task lists refer to these tiles; vmap gives
+    // every stored block its tile and column (tile * 64 + column).
+    int ex_C = 1;
+    int64_t ex_nnzb = 0;
+    std::vector<int32_t> vmap;
+    int32_t *d_vmap = nullptr;
+
     std::atomic<int64_t> reuse_count{0};
     ~Schedule();
 };
@@ -130,6 +139,8 @@ cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
 cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, void *out, cudaStream_t s);
+cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t nnzb, int R, int C, uint16_t *tiles,
+                            cudaStream_t s);
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
                              const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);

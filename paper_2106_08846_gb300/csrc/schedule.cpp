@@ -287,6 +287,39 @@ void plan_tc(Schedule &sc) {
     }
 }
 
+// Narrow bf16 blocks (R in 16..128, C in 1..8) on the tensor cores: the
+// kept blocks of each block row, grouped by 64-column tile, become dense
+// R x 64 tiles with zeros for absent blocks -- a gathered-K product whose
+// gather is replaced by zero padding. Worth it while the tiles are dense
+// enough: on average at least 8 kept columns per tile (the tensor cores do
+// 64 columns of work per tile at many times the SIMT rate; at 6.4 the two
+// paths measured about even on 1024x1024 weights at 16384 tokens). Fills the tile
+// structure (ptr, ind) and vmap; false if the shape or density does not fit.
+bool reblock_for_tc(const Schedule &sc, std::vector<int32_t> &ptr, std::vector<int32_t> &ind,
+                    std::vector<int32_t> &vmap) {
+    if (sc.dt != BSR_BF16 || !(sc.C == 1 || sc.C == 2 || sc.C == 4 || sc.C == 8) ||
+        !(sc.R == 16 || sc.R == 32 || sc.R == 64 || sc.R == 128) || sc.K % 8 != 0 || sc.nnzb == 0)
+        return false;
+    const int64_t tw = 64 / sc.C;   // block columns per tile
+    ptr.assign((size_t)sc.MB + 1, 0);
+    ind.clear();
+    vmap.assign((size_t)sc.nnzb, 0);
+    for (int64_t i = 0; i < sc.MB; i++) {
+        int64_t last = -1;
+        for (int32_t p = sc.indptr[i]; p < sc.indptr[i + 1]; p++) {
+            const int64_t t = sc.indices[p] / tw;
+            if (t != last) {
+                ind.push_back((int32_t)t);
+                last = t;
+            }
+            vmap[(size_t)p] = (int32_t)(((int64_t)ind.size() - 1) * 64 + (sc.indices[p] % tw) * sc.C);
+        }
+        ptr[(size_t)i + 1] = (int32_t)ind.size();
+        if ((int64_t)ind.size() * 64 > INT32_MAX) return false;
+    }
+    return sc.nnzb * sc.C >= 8 * (int64_t)ind.size();
+}
+
 const char *env_str(const char *name) {
     const char *v = getenv(name);
     return v && *v ? v : nullptr;
@@ -306,7 +339,29 @@ bsr_status_t build_schedule(Schedule &sc) {
     const char *force = env_str("BSR_FORCE_VARIANT");
     const bool want_generic = force && std::string(force) == "generic";
     const bool want_xstage = force && std::string(force) == "xstage";
-    if (!want_generic && !want_xstage && tc_supports(sc.R, sc.C, sc.dt, sc.K)) {
+    sc.ex_C = sc.C;
+    sc.ex_nnzb = sc.nnzb;
+    std::vector<int32_t> tptr, tind;
+    const bool reblock = !want_generic && !want_xstage && !tc_supports(sc.R, sc.C, sc.dt, sc.K) &&
+                         reblock_for_tc(sc, tptr, tind, sc.vmap);
+    if (!reblock) sc.vmap.clear();
+    if (!want_generic && !want_xstage && (reblock || tc_supports(sc.R, sc.C, sc.dt, sc.K))) {
+        // plan on the tile structure (the user's arrays stay the cache key)
+        std::vector<int32_t> uptr, uind;
+        const int uC = sc.C;
+        const int64_t unnzb = sc.nnzb, uKB = sc.KB;
+        if (reblock) {
+            uptr.swap(sc.indptr);
+            uind.swap(sc.indices);
+            sc.indptr.swap(tptr);
+            sc.indices.swap(tind);
+            sc.C = 64;
+            sc.nnzb = sc.indptr.back();
+            sc.KB = (sc.K + 63) / 64;
+            sc.ex_C = 64;
+            sc.ex_nnzb = sc.nnzb;
+            row_stats(sc);
+        }
         sc.variant = V_TC;
         sc.tn = kTcTokens;
         sc.threads = 192;
@@ -317,6 +372,13 @@ bsr_status_t build_schedule(Schedule &sc) {
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
         make_items(sc, limit, true);
         plan_tc(sc);
+        if (reblock) {
+            sc.indptr.swap(uptr);
+            sc.indices.swap(uind);
+            sc.C = uC;
+            sc.nnzb = unnzb;
+            sc.KB = uKB;
+        }
     } else if (!want_generic && xstage_supports(sc.R, sc.C, sc.dt, sc.K)) {
         sc.variant = V_XSTAGE;
         sc.tn = kXsTokens;
@@ -346,7 +408,8 @@ bsr_status_t build_schedule(Schedule &sc) {
     if (upload(&sc.d_items, sc.items) != cudaSuccess || upload(&sc.d_splits, sc.splits) != cudaSuccess ||
         upload(&sc.d_group_begin, sc.group_begin) != cudaSuccess ||
         upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess ||
-        upload(&sc.d_xs_perm, sc.xs_perm) != cudaSuccess || upload(&sc.d_xs_vdst, sc.xs_vdst) != cudaSuccess) {
+        upload(&sc.d_xs_perm, sc.xs_perm) != cudaSuccess || upload(&sc.d_xs_vdst, sc.xs_vdst) != cudaSuccess ||
+        upload(&sc.d_vmap, sc.vmap) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
@@ -362,11 +425,11 @@ bsr_status_t build_schedule(Schedule &sc) {
 bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
     const Schedule &sc = *h.sched;
-    if (sc.variant == V_TC && sc.nnzb == 0) return BSR_OK;
+    if (sc.variant == V_TC && sc.ex_nnzb == 0) return BSR_OK;
     if (sc.variant != V_XSTAGE && sc.variant != V_TC) return BSR_OK;
     // xstage: the task blobs (item tables and records from the schedule's
     // template, then this handle's block values)
-    const size_t bytes = sc.variant == V_TC ? (size_t)sc.nnzb * tc_block_bytes(sc.R, sc.C, sc.dt) : sc.xs_blob.size() * 4;
+    const size_t bytes = sc.variant == V_TC ? (size_t)sc.ex_nnzb * tc_block_bytes(sc.R, sc.ex_C, sc.dt) : sc.xs_blob.size() * 4;
     if (bytes == 0) return BSR_OK;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
@@ -375,7 +438,23 @@ bsr_status_t pack_data(Handle &h) {
     }
     cudaError_t e = cudaSuccess;
     if (sc.variant == V_TC) {
-        e = pack_tc_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, h.data_packed, 0);
+        if (sc.ex_C != sc.C) {
+            // re-blocked: zero-filled R x 64 tiles first, then the MMA layout
+            void *tiles = nullptr;
+            const size_t tbytes = (size_t)sc.ex_nnzb * sc.R * 64 * 2;
+            if (cudaMalloc(&tiles, tbytes) != cudaSuccess) {
+                cudaGetLastError();
+                return BSR_ERR_ALLOC;
+            }
+            e = cudaMemset(tiles, 0, tbytes);
+            if (e == cudaSuccess)
+                e = reblock_tc_data((const uint16_t *)h.data, sc.d_vmap, sc.nnzb, sc.R, sc.C, (uint16_t *)tiles, 0);
+            if (e == cudaSuccess) e = pack_tc_data(tiles, sc.dt, sc.ex_nnzb, sc.R, 64, h.data_packed, 0);
+            if (e == cudaSuccess) e = cudaDeviceSynchronize();
+            cudaFree(tiles);
+        } else {
+            e = pack_tc_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, h.data_packed, 0);
+        }
     } else {
         e = cudaMemcpy(h.data_packed, sc.xs_blob.data(), bytes, cudaMemcpyHostToDevice);
         if (e == cudaSuccess && sc.nnzb > 0)

@@ -453,6 +453,21 @@ __global__ void k_pack_tc_f32(const float *__restrict__ data, float *__restrict_
     }
 }
 
+// Narrow bf16 blocks into zero-filled R x 64 tiles: element (r, c) of stored
+// block p goes to tile vmap[p] / 64, row r, column vmap[p] % 64 + c.
+__global__ void k_reblock(const uint16_t *__restrict__ data, const int32_t *__restrict__ vmap, int64_t nnzb, int R,
+                          int C, uint16_t *__restrict__ tiles) {
+    const int64_t total = nnzb * R * C;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = e / ((int64_t)R * C);
+        const int rc = (int)(e - p * R * C);
+        const int r = rc / C, c = rc - r * C;
+        const int64_t v = vmap[p];
+        tiles[((v >> 6) * R + r) * 64 + (v & 63) + c] = data[e];
+    }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
@@ -499,7 +514,7 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.N = la.N;
     a.K = sc.K;
     a.M = sc.M;
-    a.C = sc.C;
+    a.C = sc.ex_C;   // the execution block width (64 for re-blocked narrow blocks)
     a.nchunks = (int)((sc.K + KC - 1) / KC);
     a.w_off = (sizeof(T) == 4 ? 2 : 1) * NS * kStageBytes;
     a.trec_smem = a.w_off + (uint32_t)((sc.tc.task_wbytes[gidx] + 15) & ~size_t(15));
@@ -577,6 +592,15 @@ cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, 
         k_pack_tc_f32<<<grid, 256, 0, s>>>(static_cast<const float *>(data), static_cast<float *>(out), nnzb, R, C);
     else
         k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), static_cast<uint16_t *>(out), nnzb, R, C);
+    return cudaGetLastError();
+}
+
+cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t nnzb, int R, int C, uint16_t *tiles,
+                            cudaStream_t s) {
+    const int64_t total = nnzb * R * C;
+    if (total == 0) return cudaSuccess;
+    const int grid = (int)std::min<int64_t>((total + 255) / 256, 1 << 20);
+    k_reblock<<<grid, 256, 0, s>>>(data, vmap, nnzb, R, C, tiles);
     return cudaGetLastError();
 }
 
