@@ -57,10 +57,6 @@ constexpr int NS = kXsStages;
 constexpr int NCW = kXsConsumerWarps;
 constexpr int WD = kXsWDup;
 constexpr int kItab = kXsItab;   // ints per item in a task's item table
-#ifndef XS_UNROLL
-#define XS_UNROLL 1
-#endif
-constexpr int kUnroll = XS_UNROLL;   // unrolling of the one-column block loop
 constexpr uint64_t kDrainNs = 200000000ull;   // bound for TMA loads already issued (they take microseconds)
 
 struct XsArgs {
@@ -241,38 +237,24 @@ __device__ __forceinline__ void item_chunk(Tile<TR> &acc, const unsigned char *s
         // group's columns fall in distinct banks), dealt round-robin to the
         // S warps of the item; lane group ks takes block ks of each group
         const int ngr = (hi - lo + NKS - 1) / NKS;
-        // (U groups per step with all loads first measured no faster: the
-        // shared-memory pipe, not one warp's dependent chain, sets the pace)
-        constexpr int U = 1;
-        for (int jg = piece; jg < ngr; jg += S * U) {
-            int lbu[U];
-            bool v[U];
-            uint32_t off[U];
-#pragma unroll
-            for (int u = 0; u < U; u++) {
-                lbu[u] = lo + (jg + S * u) * NKS + ks;
-                v[u] = jg + S * u < ngr && lbu[u] < hi;
-                if (!v[u]) lbu[u] = lo;   // a valid position: loads stay in bounds, the FMA is skipped
+        for (int jg = piece; jg < ngr; jg += S) {
+            const int lb = lo + jg * NKS + ks;
+            if (NKS > 1 && lb >= hi) continue;
+            uint32_t off;
+            f2_t wd[TR];
+            if constexpr (R == 1) {
+                // 1x1: (X offset, weight) in one 8-byte record entry
+                const int2 ow = reinterpret_cast<const int2 *>(idx)[lb];
+                off = (uint32_t)ow.x ^ tgx;
+                wd[0] = pack2(__int_as_float(ow.y), __int_as_float(ow.y));
+            } else {
+                off = (uint32_t)idx[lb] ^ tgx;
+                load_wd<TR>(wbase + lb * R * WD, wd);
             }
-            float x[U][8];
-            f2_t wd[U][TR];
+            float x[8];
 #pragma unroll
-            for (int u = 0; u < U; u++) {
-                if constexpr (R == 1) {
-                    // 1x1: (X offset, weight) in one 8-byte record entry
-                    const int2 ow = reinterpret_cast<const int2 *>(idx)[lbu[u]];
-                    off[u] = (uint32_t)ow.x ^ tgx;
-                    wd[u][0] = pack2(__int_as_float(ow.y), __int_as_float(ow.y));
-                } else {
-                    off[u] = (uint32_t)idx[lbu[u]] ^ tgx;
-                    load_wd<TR>(wbase + lbu[u] * R * WD, wd[u]);
-                }
-#pragma unroll
-                for (int i = 0; i < 8; i++) x[u][i] = ld_x(st + off[u] + i * 1024, T());
-            }
-#pragma unroll
-            for (int u = 0; u < U; u++)
-                if (v[u]) acc.fma(x[u], wd[u]);
+            for (int i = 0; i < 8; i++) x[i] = ld_x(st + off + i * 1024, T());
+            acc.fma(x, wd);
         }
         return;
     } else {
