@@ -123,6 +123,7 @@ Schedule::~Schedule() {
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);
         cudaFree(tc.d_rec_off[gi]);
+        cudaFree(tc.d_worder[gi]);
     }
     cudaFree(d_indices);
 }

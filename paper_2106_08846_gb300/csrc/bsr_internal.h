@@ -86,6 +86,7 @@ struct Schedule {
     // every stored block its tile and column (tile * 64 + column).
     int ex_C = 1;
     int64_t ex_nnzb = 0;
+    int64_t tc_w_total = 0;   // bytes of the tensor-core kernel's packed values (all task sizes)
     std::vector<int32_t> vmap;
     int32_t *d_vmap = nullptr;
 
@@ -138,7 +139,8 @@ struct LaunchArgs {
 cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
-cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, void *out, cudaStream_t s);
+cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
+                         cudaStream_t s);
 cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t nnzb, int R, int C, uint16_t *tiles,
                             cudaStream_t s);
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,

@@ -245,17 +245,20 @@ void plan_tc(Schedule &sc) {
     const int64_t es = (int64_t)dtype_size(sc.dt);
     const int64_t nch = (sc.K + kc - 1) / kc;
     const size_t per_block = tc_block_bytes(sc.R, sc.C, sc.dt);
+    int64_t total = 0;   // bytes of packed values over all usable G
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         const int G = kTcG[gi];
         std::vector<int32_t> &rec = sc.tc.rec[gi];
         std::vector<int32_t> &off = sc.tc.rec_off[gi];
+        std::vector<int32_t> &order = sc.tc.worder[gi];
         rec.clear();
         off.clear();
+        order.clear();
         size_t wmax = 0, imax = 0;
-        std::vector<std::vector<int32_t>> per_chunk((size_t)nch);
+        std::vector<std::vector<int32_t>> per_chunk((size_t)nch), src((size_t)nch);
         for (size_t t = 0; t < sc.items.size(); t += G) {
             for (auto &v : per_chunk) v.clear();
-            int32_t wblk = 0;
+            for (auto &v : src) v.clear();
             const size_t t_end = std::min(sc.items.size(), t + G);
             for (size_t k = t; k < t_end; k++) {
                 const Item &it = sc.items[k];
@@ -263,28 +266,38 @@ void plan_tc(Schedule &sc) {
                     const int64_t col = sc.indices[it.p0 + b];
                     const int64_t c = (col * sc.C) / kc;
                     const int32_t a32 = (int32_t)(((col * sc.C) % kc) * es / 32);
-                    per_chunk[(size_t)c].push_back(a32 | (int32_t)((k - t) << 2) | ((b == 0) << 7) |
-                                                   ((wblk + b) << 8));
+                    per_chunk[(size_t)c].push_back(a32 | (int32_t)((k - t) << 2) | ((b == 0) << 7));
+                    src[(size_t)c].push_back(it.p0 + b);
                 }
-                wblk += it.p1 - it.p0;
             }
             off.push_back((int32_t)rec.size());
             const size_t head = rec.size();
-            rec.resize(head + (size_t)tc_pad4(nch + 1), 0);
+            rec.resize(head + (size_t)tc_pad4(nch + 2), 0);
+            rec[head] = (int32_t)order.size();   // the task's first packed block
             int32_t n = 0;
             for (int64_t c = 0; c < nch; c++) {
-                rec[head + (size_t)c] = n;
+                rec[head + 1 + (size_t)c] = n;
                 n += (int32_t)per_chunk[(size_t)c].size();
+                wmax = std::max(wmax, per_chunk[(size_t)c].size() * per_block);
             }
-            rec[head + (size_t)nch] = n;
-            for (int64_t c = 0; c < nch; c++) rec.insert(rec.end(), per_chunk[(size_t)c].begin(), per_chunk[(size_t)c].end());
-            rec.resize(head + (size_t)tc_pad4(nch + 1) + (size_t)tc_pad4(n), 0);
-            wmax = std::max(wmax, (size_t)wblk * per_block);
+            rec[head + 1 + (size_t)nch] = n;
+            for (int64_t c = 0; c < nch; c++) {
+                rec.insert(rec.end(), per_chunk[(size_t)c].begin(), per_chunk[(size_t)c].end());
+                order.insert(order.end(), src[(size_t)c].begin(), src[(size_t)c].end());
+            }
+            rec.resize(head + (size_t)tc_pad4(nch + 2) + (size_t)tc_pad4(n), 0);
             imax = std::max(imax, (rec.size() - head) * 4);
         }
-        sc.tc.task_wbytes[gi] = wmax;
+        sc.tc.task_wbytes[gi] = (wmax + 15) & ~size_t(15);
         sc.tc.task_ibytes[gi] = imax;
+        const bool ok = G * sc.R <= kTcTmemCols &&
+                        tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], imax, sc.dt) <= (size_t)kTcMaxSmem &&
+                        (int64_t)order.size() < INT32_MAX;
+        sc.tc.w_off[gi] = ok ? (total + 255) & ~int64_t(255) : -1;
+        if (ok) total = sc.tc.w_off[gi] + (int64_t)order.size() * (int64_t)per_block;
+        else order.clear();
     }
+    sc.tc_w_total = total;
 }
 
 // Narrow bf16 blocks (R in 16..128, C in 1..8) on the tensor cores: the
@@ -365,12 +378,8 @@ bsr_status_t build_schedule(Schedule &sc) {
         sc.variant = V_TC;
         sc.tn = kTcTokens;
         sc.threads = 192;
-        const int64_t nch = (sc.K + tc_chunk_cols(sc.dt) - 1) / tc_chunk_cols(sc.dt);
-        const int64_t avail = (int64_t)tc_task_budget(sc.R, sc.dt) - 4 * xstage_pad4(nch + 1) - 16;
-        const int64_t lmax = std::max<int64_t>(1, avail / (int64_t)(tc_block_bytes(sc.R, sc.C, sc.dt) + 4));
-        int64_t limit = split_limit(sc);
-        limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
-        make_items(sc, limit, true);
+        // block values stream per chunk: only balance decides the splitting
+        make_items(sc, split_limit(sc), true);
         plan_tc(sc);
         if (reblock) {
             sc.indptr.swap(uptr);
@@ -415,7 +424,8 @@ bsr_status_t build_schedule(Schedule &sc) {
     }
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (upload(&sc.tc.d_rec[gi], sc.tc.rec[gi]) != cudaSuccess ||
-            upload(&sc.tc.d_rec_off[gi], sc.tc.rec_off[gi]) != cudaSuccess) {
+            upload(&sc.tc.d_rec_off[gi], sc.tc.rec_off[gi]) != cudaSuccess ||
+            upload(&sc.tc.d_worder[gi], sc.tc.worder[gi]) != cudaSuccess) {
             cudaGetLastError();
             return BSR_ERR_ALLOC;
         }
@@ -429,7 +439,7 @@ bsr_status_t pack_data(Handle &h) {
     if (sc.variant != V_XSTAGE && sc.variant != V_TC) return BSR_OK;
     // xstage: the task blobs (item tables and records from the schedule's
     // template, then this handle's block values)
-    const size_t bytes = sc.variant == V_TC ? (size_t)sc.ex_nnzb * tc_block_bytes(sc.R, sc.ex_C, sc.dt) : sc.xs_blob.size() * 4;
+    const size_t bytes = sc.variant == V_TC ? (size_t)sc.tc_w_total : sc.xs_blob.size() * 4;
     if (bytes == 0) return BSR_OK;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
@@ -449,11 +459,17 @@ bsr_status_t pack_data(Handle &h) {
             e = cudaMemset(tiles, 0, tbytes);
             if (e == cudaSuccess)
                 e = reblock_tc_data((const uint16_t *)h.data, sc.d_vmap, sc.nnzb, sc.R, sc.C, (uint16_t *)tiles, 0);
-            if (e == cudaSuccess) e = pack_tc_data(tiles, sc.dt, sc.ex_nnzb, sc.R, 64, h.data_packed, 0);
+            for (int gi = 0; gi < kTcTaskSizes && e == cudaSuccess; gi++)
+                if (sc.tc.w_off[gi] >= 0)
+                    e = pack_tc_data(tiles, sc.dt, sc.tc.d_worder[gi], (int64_t)sc.tc.worder[gi].size(), sc.R, 64,
+                                     (unsigned char *)h.data_packed + sc.tc.w_off[gi], 0);
             if (e == cudaSuccess) e = cudaDeviceSynchronize();
             cudaFree(tiles);
         } else {
-            e = pack_tc_data(h.data, sc.dt, sc.nnzb, sc.R, sc.C, h.data_packed, 0);
+            for (int gi = 0; gi < kTcTaskSizes && e == cudaSuccess; gi++)
+                if (sc.tc.w_off[gi] >= 0)
+                    e = pack_tc_data(h.data, sc.dt, sc.tc.d_worder[gi], (int64_t)sc.tc.worder[gi].size(), sc.R, sc.C,
+                                     (unsigned char *)h.data_packed + sc.tc.w_off[gi], 0);
         }
     } else {
         e = cudaMemcpy(h.data_packed, sc.xs_blob.data(), bytes, cudaMemcpyHostToDevice);
@@ -511,11 +527,7 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
         const char *v = getenv("BSR_TC_G");
         return v ? atoi(v) : 0;
     }();
-    auto fits = [&](int G) {
-        const int gi = tc_g_index(G);
-        return G * sc.R <= kTcTmemCols &&
-               tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt) <= (size_t)kTcMaxSmem;
-    };
+    auto fits = [&](int G) { return sc.tc.w_off[tc_g_index(G)] >= 0; };   // planned and packed for G
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (forced == kTcG[gi] && fits(forced)) return forced;
     const double kOverheadItems = 4.0;

@@ -58,7 +58,8 @@ struct TcArgs {
     int n_items, G, n_tasks;
     const int32_t *trec;      // task records: chunk starts, then MMA entries
     const int32_t *trec_off;  // per task: record offset (ints)
-    const void *wpk;          // block values in the MMA's B layout (fp32: high then low parts)
+    const void *wpk;          // block values in the MMA's B layout (fp32: high then low parts), task-chunk order
+    uint32_t wstage;          // bytes of one W ring stage
     const float *bias;
     void *Y;
     float *ws;
@@ -163,8 +164,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
     uint64_t *full = reinterpret_cast<uint64_t *>(base + a.bar_off);
     uint64_t *empty = full + NS;
     uint64_t *split = empty + NS;    // fp32: the stage's high/low parts are ready
-    uint64_t *wbar = split + NS;     // block values landed
-    uint64_t *done = wbar + 1;       // every MMA completed
+    uint64_t *done = split + NS;     // every MMA completed
     uint64_t *rbar = done + 1;       // task record landed
     int *misc = reinterpret_cast<int *>(base + a.misc_off);   // [0] abort flag, [1] TMEM address
     int *itab = misc + 4;                                     // per item: row p0 p1 slot - len
@@ -186,7 +186,6 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
             ptx::mbar_init(&empty[s], 1);
             ptx::mbar_init(&split[s], 1);
         }
-        ptx::mbar_init(wbar, 1);
         ptx::mbar_init(done, 1);
         ptx::mbar_init(rbar, 1);
         misc[0] = 0;
@@ -220,25 +219,18 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         if (lane == 0) {
             ptx::prefetch_tensormap(&xmap);
             const int32_t *trec = a.trec + __ldg(a.trec_off + task);
-            const int n_ent = __ldg(trec + nch);
-            const uint32_t rec_bytes = (uint32_t)(pad4(nch + 1) + pad4(n_ent)) * 4;
+            const int n_ent = __ldg(trec + 1 + nch);
+            const uint32_t rec_bytes = (uint32_t)(pad4(nch + 2) + pad4(n_ent)) * 4;
             ptx::mbar_arrive_expect_tx(rbar, rec_bytes);
             ptx::bulk_load(I_s, trec, rec_bytes, rbar);
-            uint32_t total = 0;
-            for (int g = 0; g < g_count; g++) total += (uint32_t)itab[6 * g + 5] * wblock;
-            ptx::mbar_arrive_expect_tx(wbar, total);
-            uint32_t woff = 0;
             const unsigned char *wsrc = static_cast<const unsigned char *>(a.wpk);
-            for (int g = 0; g < g_count; g++) {
-                const int len = itab[6 * g + 5];
-                if (len) ptx::bulk_load(W_s + woff, wsrc + (int64_t)itab[6 * g + 1] * wblock, len * wblock, wbar);
-                woff += len * wblock;
-            }
             int k = 0;          // ring slots used (chunks with work, in order)
             int stalled = -1;   // test hook: the slot left empty
             bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);   // chunk starts, from shared memory
+            const int64_t wfirst = ok ? I_s[0] : 0;                   // the task's first packed block
             for (int c = 0; ok && c < nch; c++) {
-                if (I_s[c] == I_s[c + 1]) continue;   // no block of this task in chunk c
+                const int lo = I_s[1 + c], hi = I_s[2 + c];
+                if (lo == hi) continue;   // no block of this task in chunk c
                 const int s = k % NS;
                 if (k >= NS && !ptx::mbar_wait_bounded(&empty[s], ((k / NS) - 1) & 1, a.wait_ns)) {
                     ok = false;
@@ -249,8 +241,11 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                     stalled = k++;
                     continue;
                 }
-                ptx::mbar_arrive_expect_tx(&full[s], kStageBytes);
+                // the X chunk and, beside it, the task's block values for this chunk
+                const uint32_t wbytes = (uint32_t)(hi - lo) * wblock;
+                ptx::mbar_arrive_expect_tx(&full[s], kStageBytes + wbytes);
                 ptx::tma_load_2d(base + s * kStageBytes, &xmap, c * TcCfg<T>::KC, (int32_t)n0, &full[s]);
+                ptx::bulk_load(W_s + s * a.wstage, wsrc + (wfirst + lo) * wblock, wbytes, &full[s]);
                 k++;
             }
             if (!ok) {
@@ -259,19 +254,16 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
             }
             for (int d = max(0, k - NS); d < k; d++)
                 if (d != stalled) ptx::mbar_wait_bounded(&full[d % NS], (d / NS) & 1, kDrainNs);
-            ptx::mbar_wait_bounded(wbar, 0, kDrainNs);
             ptx::mbar_wait_bounded(rbar, 0, kDrainNs);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer
         if (lane == 0) {
-            bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns) && ptx::mbar_wait_bounded(wbar, 0, a.wait_ns) &&
-                      !aborted(misc);
-            const uint32_t w_base = ptx::smem_addr(W_s);
-            const int32_t *ent = I_s + pad4(nch + 1);
+            bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns) && !aborted(misc);
+            const int32_t *ent = I_s + pad4(nch + 2);
             int k = 0;   // chunks consumed
             for (int c = 0; ok && c < nch; c++) {
-                const int lo = I_s[c], hi = I_s[c + 1];
+                const int lo = I_s[1 + c], hi = I_s[2 + c];
                 if (lo == hi) continue;
                 const int s = k % NS;
                 // fp32: wait for the split parts (the split warps waited for the copy)
@@ -281,11 +273,12 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                 }
                 tc_fence_after();
                 const uint32_t stage = ptx::smem_addr(base + s * kStageBytes);
+                const uint32_t w_stage = ptx::smem_addr(W_s + s * a.wstage);
                 for (int e = lo; e < hi; e++) {
                     const uint32_t v = (uint32_t)ent[e];
                     const uint32_t a_row = stage + (v & 3u) * 32u;
                     const uint32_t g = (v >> 2) & 31u, first = (v >> 7) & 1u;
-                    const uint32_t w_blk = w_base + (v >> 8) * wblock;
+                    const uint32_t w_blk = w_stage + (uint32_t)(e - lo) * wblock;
                     if constexpr (F32) {
                         // 3xTF32: high x high + high x low + low x high, K = 8 per MMA
                         constexpr uint32_t idesc = idesc_tf32(TN, R);
@@ -334,7 +327,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
             split_ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);
             int k = 0;
             for (int c = 0; split_ok && c < nch; c++) {
-                if (I_s[c] == I_s[c + 1]) continue;
+                if (I_s[1 + c] == I_s[2 + c]) continue;
                 const int s = k % NS;
                 const bool got = ptx::mbar_wait_bounded(&full[s], (k / NS) & 1, a.wait_ns) && !aborted(misc);
                 if (ptx::named_barrier_or(2, 128, !got)) { split_ok = false; break; }
@@ -424,29 +417,32 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
 // Block values into the MMA's B operand layout (K-major, no swizzle): for each
 // K-slice of 16 columns, 8-row x 16-byte core matrices, 128 bytes apart along
 // K and 256 bytes apart along the rows.
-__global__ void k_pack_tc(const uint16_t *__restrict__ data, uint16_t *__restrict__ out, int64_t nnzb, int R, int C) {
-    const int64_t total = nnzb * R * C;
+// Packed block i holds stored block order[i].
+__global__ void k_pack_tc(const uint16_t *__restrict__ data, const int32_t *__restrict__ order,
+                          uint16_t *__restrict__ out, int64_t n, int R, int C) {
+    const int64_t total = n * R * C;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
          e += (int64_t)gridDim.x * blockDim.x) {
         const int64_t p = e / ((int64_t)R * C);
         const int rc = (int)(e - p * R * C);
-        const int n = rc / C, k = rc - n * C;
-        const int64_t dst = p * R * C + (k >> 4) * (R * 16) + (n >> 3) * 128 + ((k & 15) >> 3) * 64 + (n & 7) * 8 + (k & 7);
-        out[dst] = data[e];
+        const int n_ = rc / C, k = rc - n_ * C;
+        const int64_t dst = p * R * C + (k >> 4) * (R * 16) + (n_ >> 3) * 128 + ((k & 15) >> 3) * 64 + (n_ & 7) * 8 + (k & 7);
+        out[dst] = data[(int64_t)order[p] * R * C + rc];
     }
 }
 
 // fp32 block values as two tf32 B operands, high part then low part, each in
 // the layout above with 8-column K-slices of 8-row x 16-byte core matrices.
-__global__ void k_pack_tc_f32(const float *__restrict__ data, float *__restrict__ out, int64_t nnzb, int R, int C) {
-    const int64_t total = nnzb * R * C;
+__global__ void k_pack_tc_f32(const float *__restrict__ data, const int32_t *__restrict__ order,
+                              float *__restrict__ out, int64_t n, int R, int C) {
+    const int64_t total = n * R * C;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
          e += (int64_t)gridDim.x * blockDim.x) {
         const int64_t p = e / ((int64_t)R * C);
         const int rc = (int)(e - p * R * C);
-        const int n = rc / C, k = rc - n * C;
-        const int64_t at = p * R * C * 2 + (k >> 3) * (R * 8) + (n >> 3) * 64 + ((k & 7) >> 2) * 32 + (n & 7) * 4 + (k & 3);
-        const float w = data[e];
+        const int n_ = rc / C, k = rc - n_ * C;
+        const int64_t at = p * R * C * 2 + (k >> 3) * (R * 8) + (n_ >> 3) * 64 + ((k & 7) >> 2) * 32 + (n_ & 7) * 4 + (k & 3);
+        const float w = data[(int64_t)order[p] * R * C + rc];
         const float h = __uint_as_float(__float_as_uint(w) & 0xffffe000u);
         out[at] = h;
         out[at + (int64_t)R * C] = w - h;
@@ -506,7 +502,9 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.n_tasks = (n_items + G - 1) / G;
     a.trec = sc.tc.d_rec[gidx];
     a.trec_off = sc.tc.d_rec_off[gidx];
-    a.wpk = la.data;
+    if (sc.tc.w_off[gidx] < 0) return cudaErrorInvalidConfiguration;
+    a.wpk = static_cast<const unsigned char *>(la.data) + sc.tc.w_off[gidx];
+    a.wstage = (uint32_t)sc.tc.task_wbytes[gidx];
     a.bias = la.bias;
     a.Y = la.Y;
     a.ws = la.ws;
@@ -517,10 +515,10 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.C = sc.ex_C;   // the execution block width (64 for re-blocked narrow blocks)
     a.nchunks = (int)((sc.K + KC - 1) / KC);
     a.w_off = (sizeof(T) == 4 ? 2 : 1) * NS * kStageBytes;
-    a.trec_smem = a.w_off + (uint32_t)((sc.tc.task_wbytes[gidx] + 15) & ~size_t(15));
+    a.trec_smem = a.w_off + NS * a.wstage;
     a.bias_off = a.trec_smem + (uint32_t)((sc.tc.task_ibytes[gidx] + 15) & ~size_t(15));
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * R * 4 + 15) & ~size_t(15));
-    a.misc_off = a.bar_off + (3 * NS + 3) * 8;
+    a.misc_off = a.bar_off + (3 * NS + 2) * 8;
     a.tmem_cols = tmem_cols_for(G * R);
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
@@ -570,11 +568,11 @@ int tc_g_index(int G) {
     return 0;
 }
 
-size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt) {
+size_t tc_smem_bytes(int R, int G, size_t wstage, size_t ibytes, bsr_dtype_t dt) {
     const size_t ring = dt == BSR_F32 ? (size_t)2 * kTcStagesF32 * kStageBytes : (size_t)kTcStages * kStageBytes;
     const int ns = dt == BSR_F32 ? kTcStagesF32 : kTcStages;
-    return ring + ((wbytes + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
-           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (3 * ns + 3) * 8 + (4 + 6 * 32) * 4 + 1024;
+    return ring + ns * ((wstage + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
+           (((size_t)G * R * 4 + 15) & ~size_t(15)) + (3 * ns + 2) * 8 + (4 + 6 * 32) * 4 + 1024;
 }
 
 size_t tc_task_budget(int R, bsr_dtype_t dt) {
@@ -584,14 +582,15 @@ size_t tc_task_budget(int R, bsr_dtype_t dt) {
 
 uint32_t tc_block_offset(int kk) { return (uint32_t)kk * 2; }
 
-cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, int64_t nnzb, int R, int C, void *out, cudaStream_t s) {
-    const int64_t total = nnzb * R * C;
+cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
+                         cudaStream_t s) {
+    const int64_t total = n * R * C;
     if (total == 0) return cudaSuccess;
     const int grid = (int)std::min<int64_t>((total + 255) / 256, 1 << 20);
     if (dt == BSR_F32)
-        k_pack_tc_f32<<<grid, 256, 0, s>>>(static_cast<const float *>(data), static_cast<float *>(out), nnzb, R, C);
+        k_pack_tc_f32<<<grid, 256, 0, s>>>(static_cast<const float *>(data), order, static_cast<float *>(out), n, R, C);
     else
-        k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), static_cast<uint16_t *>(out), nnzb, R, C);
+        k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), order, static_cast<uint16_t *>(out), n, R, C);
     return cudaGetLastError();
 }
 

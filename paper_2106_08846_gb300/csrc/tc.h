@@ -18,22 +18,29 @@ constexpr int kTcTmemCols = 512;       // accumulator columns per SM
 constexpr int kTcTaskSizes = 6;
 constexpr int kTcG[kTcTaskSizes] = {1, 2, 4, 8, 16, 32};
 
-// Per task size G: the task records the kernel bulk-copies (see below), and
-// the largest block-value / record footprint of a task.
+// Per task size G: the task records the kernel bulk-copies (see below), the
+// W stage (largest block-value footprint of one task's chunk) and record
+// footprints, and the order in which the block values of all tasks are
+// packed for G: task by task, chunk by chunk, in entry order, so that the
+// values one chunk of one task needs are one contiguous range (streamed
+// through a ring beside X instead of held for the whole kernel).
 struct TcPlan {
-    size_t task_wbytes[kTcTaskSizes] = {0, 0, 0, 0, 0, 0};
-    size_t task_ibytes[kTcTaskSizes] = {0, 0, 0, 0, 0, 0};
+    size_t task_wbytes[kTcTaskSizes] = {};   // W ring stage bytes
+    size_t task_ibytes[kTcTaskSizes] = {};
     std::vector<int32_t> rec[kTcTaskSizes];       // all task records of this G
     std::vector<int32_t> rec_off[kTcTaskSizes];   // per task: offset (ints, multiple of 4)
-    int32_t *d_rec[kTcTaskSizes] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
-    int32_t *d_rec_off[kTcTaskSizes] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+    std::vector<int32_t> worder[kTcTaskSizes];    // per packed block: the (execution) block it holds
+    int64_t w_off[kTcTaskSizes] = {};             // byte offset of G's packed values (-1: G not usable)
+    int32_t *d_rec[kTcTaskSizes] = {};
+    int32_t *d_rec_off[kTcTaskSizes] = {};
+    int32_t *d_worder[kTcTaskSizes] = {};
 };
 
-// A task record (int32): [ per K chunk c = 0..nchunks: index of the chunk's
-// first entry, padded to 4 | one entry per MMA-block, chunk by chunk, padded
-// to 4 ]. Entry bits: [0,2) stage column offset / 32 bytes, [2,7) item in
-// the task, 7 first block of its item, [8,32) block index in the task's
-// block values.
+// A task record (int32): [ the task's first packed block, then per K chunk
+// c = 0..nchunks the index of the chunk's first entry, padded to 4 | one
+// entry per MMA-block, chunk by chunk, padded to 4 ]. Entry e uses packed
+// block (first + e). Entry bits: [0,2) stage column offset / 32 bytes,
+// [2,7) item in the task, 7 first block of its item.
 inline int64_t tc_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
 bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K);
