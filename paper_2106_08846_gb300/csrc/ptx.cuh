@@ -60,6 +60,18 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity
     }
 }
 
+// As mbar_wait_bounded, for waits expected to be long: sleeps between
+// polls so the waiting warps leave the schedulers to the warps doing work.
+__device__ __forceinline__ bool mbar_wait_bounded_idle(uint64_t *bar, uint32_t parity, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    while (true) {
+        __nanosleep(500);
+        if (mbar_try_wait(bar, parity)) return true;
+        if (globaltimer() - t0 > limit_ns) return false;
+    }
+}
+
 // 2-D TMA tile load into shared memory, completion counted on `bar`.
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x, int32_t y,
                                            uint64_t *bar) {

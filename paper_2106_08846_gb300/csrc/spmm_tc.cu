@@ -274,33 +274,34 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                 tc_fence_after();
                 const uint32_t stage = ptx::smem_addr(base + s * kStageBytes);
                 const uint32_t w_stage = ptx::smem_addr(W_s + s * a.wstage);
+                // descriptors of the stage's first A row and first B block: an
+                // operand's descriptor is these plus its byte offset / 16 in the
+                // address field (no carry out: shared addresses stay below 256 KB)
+                const uint64_t a0 = umma_desc(stage, 16, 1024, 2), b0 = umma_desc(w_stage, 128, 256, 0);
+                const uint32_t wb16 = wblock >> 4;
                 for (int e = lo; e < hi; e++) {
                     const uint32_t v = (uint32_t)ent[e];
-                    const uint32_t a_row = stage + (v & 3u) * 32u;
                     const uint32_t g = (v >> 2) & 31u, first = (v >> 7) & 1u;
-                    const uint32_t w_blk = w_stage + (uint32_t)(e - lo) * wblock;
+                    const uint64_t ad = a0 + (uint64_t)((v & 3u) * 2u);             // + (v & 3) * 32 bytes
+                    const uint64_t bd = b0 + (uint64_t)((uint32_t)(e - lo) * wb16);
+                    const uint32_t d = tmem + g * R;
                     if constexpr (F32) {
                         // 3xTF32: high x high + high x low + low x high, K = 8 per MMA
                         constexpr uint32_t idesc = idesc_tf32(TN, R);
-                        const uint32_t a_lo = a_row + NS * kStageBytes, w_lo = w_blk + (uint32_t)R * C * 4;
+                        const uint64_t adl = ad + (uint64_t)(NS * kStageBytes >> 4), bdl = bd + (uint64_t)((uint32_t)R * C * 4 >> 4);
 #pragma unroll 2
                         for (int sl = 0; sl < C / 8; sl++) {
-                            const uint64_t ah = umma_desc(a_row + sl * 32, 16, 1024, 2);
-                            const uint64_t al = umma_desc(a_lo + sl * 32, 16, 1024, 2);
-                            const uint64_t bh = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
-                            const uint64_t bl = umma_desc(w_lo + sl * (R * 32), 128, 256, 0);
-                            mma_tf32(tmem + g * R, ah, bh, idesc, (first == 0u) | (sl > 0));
-                            mma_tf32(tmem + g * R, ah, bl, idesc, 1u);
-                            mma_tf32(tmem + g * R, al, bh, idesc, 1u);
+                            const uint64_t ka = (uint64_t)(sl * 2), kb = (uint64_t)(sl * (R * 2));   // 32 and R*32 bytes
+                            mma_tf32(d, ad + ka, bd + kb, idesc, (first == 0u) | (sl > 0));
+                            mma_tf32(d, ad + ka, bdl + kb, idesc, 1u);
+                            mma_tf32(d, adl + ka, bd + kb, idesc, 1u);
                         }
                     } else {
                         constexpr uint32_t idesc = idesc_bf16(TN, R);
 #pragma unroll 4
-                        for (int sl = 0; sl < C / 16; sl++) {
-                            const uint64_t ad = umma_desc(a_row + sl * 32, 16, 1024, 2);
-                            const uint64_t bd = umma_desc(w_blk + sl * (R * 32), 128, 256, 0);
-                            mma_bf16(tmem + g * R, ad, bd, idesc, (first == 0u) | (sl > 0));
-                        }
+                        for (int sl = 0; sl < C / 16; sl++)
+                            mma_bf16(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
+                                     (first == 0u) | (sl > 0));
                     }
                 }
                 mma_commit(&empty[s]);   // the stage is free once these MMAs completed
@@ -354,7 +355,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         ptx::named_barrier(1, 128);
         // the last commit fires after the whole main loop: allow it every chunk's bound
         const uint64_t limit = a.wait_ns * (uint64_t)(nch + 2);
-        const bool got = ptx::mbar_wait_bounded(done, 0, limit);
+        const bool got = ptx::mbar_wait_bounded_idle(done, 0, limit);   // the whole main loop: sleep while waiting
         tc_fence_after();
         const bool stop = ptx::named_barrier_or(1, 128, !got || !split_ok || aborted(misc));
         if (!got && et == 0) set_status(a.status, DEV_TIMEOUT);
