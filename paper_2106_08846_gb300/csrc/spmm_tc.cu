@@ -279,7 +279,31 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                 // address field (no carry out: shared addresses stay below 256 KB)
                 const uint64_t a0 = umma_desc(stage, 16, 1024, 2), b0 = umma_desc(w_stage, 128, 256, 0);
                 const uint32_t wb16 = wblock >> 4;
-                for (int e = lo; e < hi; e++) {
+                int e = lo;
+                if constexpr (!F32) {
+                    if (C == 16) {
+                        // one MMA per block: read and decode 4 entries, then
+                        // issue their MMAs back to back (one thread issues,
+                        // so the decoding would otherwise sit between MMAs)
+                        constexpr uint32_t idesc = idesc_bf16(TN, R);
+                        for (; e + 4 <= hi; e += 4) {
+                            const uint32_t vv[4] = {(uint32_t)ent[e], (uint32_t)ent[e + 1], (uint32_t)ent[e + 2],
+                                                    (uint32_t)ent[e + 3]};
+                            uint64_t adv[4], bdv[4];
+                            uint32_t dv[4], acc[4];
+#pragma unroll
+                            for (int j = 0; j < 4; j++) {
+                                adv[j] = a0 + (uint64_t)((vv[j] & 3u) * 2u);
+                                bdv[j] = b0 + (uint64_t)((uint32_t)(e + j - lo) * wb16);
+                                dv[j] = tmem + ((vv[j] >> 2) & 31u) * R;
+                                acc[j] = ((vv[j] >> 7) & 1u) == 0u;
+                            }
+#pragma unroll
+                            for (int j = 0; j < 4; j++) mma_bf16(dv[j], adv[j], bdv[j], idesc, acc[j]);
+                        }
+                    }
+                }
+                for (; e < hi; e++) {
                     const uint32_t v = (uint32_t)ent[e];
                     const uint32_t g = (v >> 2) & 31u, first = (v >> 7) & 1u;
                     const uint64_t ad = a0 + (uint64_t)((v & 3u) * 2u);             // + (v & 3) * 32 bytes
@@ -298,10 +322,14 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
                         }
                     } else {
                         constexpr uint32_t idesc = idesc_bf16(TN, R);
+                        if (C == 16) {   // (one MMA per block: handled in batches below)
+                            mma_bf16(d, ad, bd, idesc, first == 0u);
+                        } else {
 #pragma unroll 4
-                        for (int sl = 0; sl < C / 16; sl++)
-                            mma_bf16(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
-                                     (first == 0u) | (sl > 0));
+                            for (int sl = 0; sl < C / 16; sl++)
+                                mma_bf16(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
+                                         (first == 0u) | (sl > 0));
+                        }
                     }
                 }
                 mma_commit(&empty[s]);   // the stage is free once these MMAs completed
