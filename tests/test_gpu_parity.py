@@ -354,3 +354,36 @@ def test_sparse_narrow_bf16_blocks_stay_simt():
     h, _, Y = _run(w, X)
     assert h.schedule()["variant"] == "xstage"
     check_product(Y, oracle.bsr_from_dense(w.W, 32, 1), X, w.bias, 256)
+
+
+@pytest.mark.parametrize("R,C,dtype", [(32, 1, "f32"), (1, 1, "f32"), (16, 16, "bf16"), (32, 32, "f32")])
+def test_spmm_captured_in_cuda_graph(R, C, dtype):
+    """After bsr_reserve, bsr_spmm allocates nothing and synchronises nothing,
+    so it can be captured in a CUDA graph: replays with new X match the oracle
+    (the weight has split rows, so the split-row workspace is in the graph)."""
+    M, K, N = 256, 512, 200
+    MB, KB = M // R, K // C
+    cnt = np.full(MB, max(1, KB // 10), dtype=np.int64)
+    cnt[[1, MB // 2]] = KB   # long rows: split pieces and the reduce pass
+    w = synth.make_weight("g", 900 + R + C, M, K, R, C, dtype, 0,
+                          mask=synth.mask_from_row_counts(900 + R + C, cnt, KB))
+    bsr = _bsr()
+    h = bsr.bsr_create(*build_on_gpu(w.W, R, C), R, C, M, K)
+    h.reserve(N)
+    X0 = synth.activations(901, N, K, dtype)
+    Xd = to_dev(X0)
+    b = to_dev(w.bias)
+    Y = torch.empty((N, M), device="cuda", dtype=Xd.dtype)
+    bsr.bsr_spmm(h, Xd, b, Y, N)   # first call outside the capture (one-time kernel set-up)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        bsr.bsr_spmm(h, Xd, b, Y, N, torch.cuda.current_stream())
+    ref = oracle.bsr_from_dense(w.W, R, C)
+    for seed in (902, 903):
+        X = synth.activations(seed, N, K, dtype)
+        Xd.copy_(to_dev(X))
+        g.replay()
+        torch.cuda.synchronize()
+        assert h.check_device_status() == 0
+        check_product(to_host(Y), ref, X, w.bias, M)
