@@ -58,10 +58,23 @@ void make_items(Schedule &sc, int64_t limit, bool drop_empty = false) {
         }
         sc.splits.push_back(s);
     }
-    // One-row blocks keep row order: their tasks are many short rows, which
-    // averages out length differences, and consecutive rows let a task store
-    // whole row segments of Y.
-    if (sc.R == 1) return;
+    // One-row blocks keep rows close together: a task's rows then share the
+    // cache lines of Y its output pass writes. Inside each group of twice the
+    // consumer warps (a task of two rows per warp), the longest row is paired
+    // with the shortest, the second longest with the second shortest, and so
+    // on: warp w owns positions 2w and 2w + 1, so its work is about the mean.
+    if (sc.R == 1) {
+        const size_t grp = 2 * kXsConsumerWarpsR1;
+        std::vector<Item> g;
+        for (size_t at = 0; at < sc.items.size(); at += grp) {
+            const size_t n = std::min(grp, sc.items.size() - at);
+            g.assign(sc.items.begin() + (int64_t)at, sc.items.begin() + (int64_t)(at + n));
+            std::stable_sort(g.begin(), g.end(), [](const Item &a, const Item &b) { return a.p1 - a.p0 > b.p1 - b.p0; });
+            for (size_t k = 0; k < n; k++)
+                sc.items[at + k] = k % 2 == 0 ? g[k / 2] : g[n - 1 - k / 2];
+        }
+        return;
+    }
     std::stable_sort(sc.items.begin(), sc.items.end(),
                      [](const Item &a, const Item &b) { return a.p1 - a.p0 > b.p1 - b.p0; });
 }

@@ -322,12 +322,39 @@ __device__ __forceinline__ void reduce_tile(const Tile<TR> &acc, float (&v)[8][T
         }
 }
 
-// Item gi's finished tile: + bias, converted, to Y; or, for a piece of a
-// split row, the fp32 partial to its workspace slot.
+// A lane's reduced 8 x TR tile into slot `slot` of the token-major slot
+// array ([t][slot][r], token pitch P floats). All NKS lanes of a token group
+// hold the same sums; lane ks writes tokens i = ks mod NKS.
+template <int TR, int NRG, int P>
+__device__ __forceinline__ void write_slot(float *slots, int slot, const float (&v)[8][TR], int tg, int rg, int ks) {
+    constexpr int R = TR * NRG;
+    constexpr int NKS = 4 / NRG;
+    float *base = slots + slot * R + rg * TR;
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+        if (i % NKS != ks) continue;
+        float *dst = base + (tg + 8 * i) * P;
+        if constexpr (TR % 4 == 0) {
+#pragma unroll
+            for (int j = 0; j < TR; j += 4)
+                *reinterpret_cast<float4 *>(dst + j) = make_float4(v[i][j], v[i][j + 1], v[i][j + 2], v[i][j + 3]);
+        } else if constexpr (TR == 2) {
+            *reinterpret_cast<float2 *>(dst) = make_float2(v[i][0], v[i][1]);
+        } else {
+            dst[0] = v[i][0];
+        }
+    }
+}
+
+// Item gi's finished tile straight from the registers of the one warp that
+// owns it: + bias, converted, to Y; or, for a piece of a split row, the fp32
+// partial to its workspace slot. The NKS lanes of a token group hold the
+// same sums; lane ks stores tokens i = ks mod NKS.
 template <typename T, int TR, int NRG>
 __device__ __forceinline__ void store_tile(const XsArgs &a, const Shared &sh, const float (&v)[8][TR], int gi,
-                                           int64_t n0, int rg, int tg) {
+                                           int64_t n0, int rg, int tg, int ks) {
     constexpr int R = TR * NRG;
+    constexpr int NKS = 4 / NRG;
     const int row = sh.itab[kItab * gi + 0], slot = sh.itab[kItab * gi + 3];
     const int64_t m = (int64_t)row * R + rg * TR;
     float b[TR];
@@ -336,7 +363,7 @@ __device__ __forceinline__ void store_tile(const XsArgs &a, const Shared &sh, co
 #pragma unroll
     for (int i = 0; i < 8; i++) {
         const int64_t n = n0 + tg + 8 * i;
-        if (n >= a.N) continue;
+        if (i % NKS != ks || n >= a.N) continue;
         if (slot < 0) {
             T *dst = reinterpret_cast<T *>(a.Y) + n * a.M + m;
             if constexpr (sizeof(T) == 4 && TR % 4 == 0) {
@@ -365,6 +392,87 @@ __device__ __forceinline__ void store_tile(const XsArgs &a, const Shared &sh, co
     }
 }
 
+// Output pass, after every consumer warp wrote its slot: item g's tile is
+// the sum of the S slots g*S .. g*S+S-1 in piece order (a fixed order, so
+// results repeat bit for bit) plus the bias; converted and stored to Y, or,
+// for a piece of a split row, the fp32 partial to its workspace slot. Lanes
+// take VW-wide vectors along the task's outputs and warps take tokens (TPW
+// each, loaded together so their shared-memory latencies overlap), so each
+// store instruction writes whole row segments of Y.
+template <typename T, int R, int NW, int P>
+__device__ __forceinline__ void output_pass(const XsArgs &a, const Shared &sh, const float *slots, int S,
+                                            int g_count, int64_t n0, int warp, int lane) {
+    constexpr int VW = R >= 4 ? 4 : R;   // outputs per vector
+    constexpr int VPI = R / VW;          // vectors per item and token
+    constexpr int TPW = (TN + NW - 1) / NW;
+    const int nvec = g_count * VPI;
+    for (int c = lane; c < nvec; c += 32) {
+        const int g = c / VPI, r = (c - g * VPI) * VW;
+        const int row = sh.itab[kItab * g + 0], wslot = sh.itab[kItab * g + 3];
+        float y[TPW][VW];
+#pragma unroll
+        for (int k = 0; k < TPW; k++)
+#pragma unroll
+            for (int v = 0; v < VW; v++) y[k][v] = 0.f;
+        const float *src = slots + (g * S) * R + r;
+        for (int pc = 0; pc < S; pc++, src += R) {
+#pragma unroll
+            for (int k = 0; k < TPW; k++) {
+                const int t = warp + k * NW;
+                if (TN % NW != 0 && t >= TN) continue;
+                const float *q = src + t * P;
+                if constexpr (VW == 4) {
+                    const float4 q4 = *reinterpret_cast<const float4 *>(q);
+                    y[k][0] += q4.x;
+                    y[k][1] += q4.y;
+                    y[k][2] += q4.z;
+                    y[k][3] += q4.w;
+                } else if constexpr (VW == 2) {
+                    const float2 q2 = *reinterpret_cast<const float2 *>(q);
+                    y[k][0] += q2.x;
+                    y[k][1] += q2.y;
+                } else {
+                    y[k][0] += *q;
+                }
+            }
+        }
+        float b[VW];
+#pragma unroll
+        for (int v = 0; v < VW; v++) b[v] = wslot >= 0 ? 0.f : sh.B[g * R + r + v];
+#pragma unroll
+        for (int k = 0; k < TPW; k++) {
+            const int t = warp + k * NW;
+            const int64_t n = n0 + t;
+            if ((TN % NW != 0 && t >= TN) || n >= a.N) continue;
+            if (wslot >= 0) {
+                float *dst = a.ws + ((int64_t)wslot * a.N + n) * R + r;
+#pragma unroll
+                for (int v = 0; v < VW; v++) dst[v] = y[k][v];
+                continue;
+            }
+            float o[VW];
+#pragma unroll
+            for (int v = 0; v < VW; v++) o[v] = y[k][v] + b[v];
+            T *dst = reinterpret_cast<T *>(a.Y) + n * a.M + (int64_t)row * R + r;
+            if constexpr (sizeof(T) == 4 && VW == 4) {
+                *reinterpret_cast<float4 *>(dst) = make_float4(o[0], o[1], o[2], o[3]);
+            } else if constexpr (sizeof(T) == 4 && VW == 2) {
+                *reinterpret_cast<float2 *>(dst) = make_float2(o[0], o[1]);
+            } else if constexpr (sizeof(T) == 2 && VW == 4) {
+                uint2 pk;
+                pk.x = (uint32_t)from_f32<T>(o[0]) | ((uint32_t)from_f32<T>(o[1]) << 16);
+                pk.y = (uint32_t)from_f32<T>(o[2]) | ((uint32_t)from_f32<T>(o[3]) << 16);
+                *reinterpret_cast<uint2 *>(dst) = pk;
+            } else if constexpr (sizeof(T) == 2 && VW == 2) {
+                *reinterpret_cast<uint32_t *>(dst) =
+                    (uint32_t)from_f32<T>(o[0]) | ((uint32_t)from_f32<T>(o[1]) << 16);
+            } else {
+                dst[0] = from_f32<T>(o[0]);
+            }
+        }
+    }
+}
+
 // NW consumer warps. RW == 1: S = NW/G warps share each item (block-strided)
 // and a pairwise tree sums them. RW > 1 (G = NW RW): each warp owns RW
 // whole items, with one register tile each, and needs no tree.
@@ -387,9 +495,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         }
     }
     ptx::named_barrier(1, NW * 32);
-    // the bias, needed only by the epilogue (waited for there), and whether
-    // the task covers consecutive whole rows (then the epilogue stores whole
-    // row segments of Y)
+    // the bias, needed only by the output pass (waited for there)
     for (int e = ctid; e < g_count * R; e += NW * 32) {
         const int g = e / R, r = e - g * R;
         if (a.bias)
@@ -397,9 +503,10 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         else
             sh.B[e] = 0.f;
     }
-    if (ctid < g_count && (sh.itab[kItab * ctid + 0] != sh.itab[0] + ctid || sh.itab[kItab * ctid + 3] >= 0))
-        sh.misc[3] = 0;
     bool ok = true;
+    float *slots = reinterpret_cast<float *>(sh.base);   // the ring, free once every warp is past it
+    constexpr int PRW = xstage_slot_pitch(R, NW * RW);   // token pitch of the slots: one per item (RW > 1)
+    constexpr int PS = xstage_slot_pitch(R, NW);         // one per warp
 
     const int q = lane >> 3, tg = lane & 7;
     const int rg = q % NRG, ks = q / NRG;
@@ -438,37 +545,15 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         }
         ptx::cp_async_wait_all();   // the bias
         if (ptx::named_barrier_or(1, NW * 32, !ok || aborted(sh.misc))) return;
-        if (R == 1 && sh.misc[3]) {
-            // consecutive rows row0 .. row0+G-1: transpose the tiles through
-            // shared memory (the ring is free) and store Y row segments
-            const int PG = g_count + 1;
-            float *P = reinterpret_cast<float *>(sh.base);
-#pragma unroll
-            for (int r = 0; r < RW; r++) {
-                const int gi = warp * RW + r;
-                float v[8][TR];
-                reduce_tile<TR, NRG>(acc[r], v);
-                if (gi < g_count && ks == 0)
-#pragma unroll
-                    for (int i = 0; i < 8; i++) P[(tg + 8 * i) * PG + gi] = v[i][0];
-            }
-            ptx::named_barrier(1, NW * 32);
-            const int64_t row0 = sh.itab[0];
-            for (int e = ctid; e < TN * g_count; e += NW * 32) {
-                const int t = e / g_count, j = e - t * g_count;
-                const int64_t n = n0 + t;
-                if (n < a.N)
-                    reinterpret_cast<T *>(a.Y)[n * a.M + row0 + j] = from_f32<T>(P[t * PG + j] + sh.B[j]);
-            }
-            return;
-        }
 #pragma unroll
         for (int r = 0; r < RW; r++) {
             const int gi = warp * RW + r;
             float v[8][TR];
             reduce_tile<TR, NRG>(acc[r], v);
-            if (gi < g_count && ks == 0) store_tile<T, TR, NRG>(a, sh, v, gi, n0, rg, tg);
+            if (gi < g_count) write_slot<TR, NRG, PRW>(slots, gi, v, tg, rg, ks);
         }
+        ptx::named_barrier(1, NW * 32);
+        output_pass<T, R, NW, PRW>(a, sh, slots, 1, g_count, n0, warp, lane);
         return;
     }
 
@@ -506,58 +591,21 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     // verdict is the same for all of them (barrier reduction)
     ptx::cp_async_wait_all();   // the bias
     if (ptx::named_barrier_or(1, NW * 32, !ok || aborted(sh.misc))) return;
-    // pairwise tree over the S warps of each item: in round `step`, the warp
-    // of piece p (p % 2step == step) hands its tile to piece p - step
-    constexpr int PS = R + 4;          // padded row of a tile in shared memory (16-byte aligned)
-    float *P = reinterpret_cast<float *>(sh.base);
-    const int half = (S + 1) / 2;      // tiles per item in the first round
-    for (int step = 1; step < S; step <<= 1) {
-        float *slot = P + (gi * half + piece / (2 * step)) * TN * PS;
-        if (has_item && piece % (2 * step) == step && ks == 0) {
-#pragma unroll
-            for (int i = 0; i < 8; i++) {
-                float *dst = slot + (tg + 8 * i) * PS + rg * TR;
-                if constexpr (TR % 4 == 0) {
-#pragma unroll
-                    for (int j = 0; j < TR; j += 4)
-                        *reinterpret_cast<float4 *>(dst + j) = make_float4(v[i][j], v[i][j + 1], v[i][j + 2], v[i][j + 3]);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < TR; j++) dst[j] = v[i][j];
-                }
-            }
-        }
-        ptx::named_barrier(1, NW * 32);
-        if (has_item && piece % (2 * step) == 0 && piece + step < S) {
-#pragma unroll
-            for (int i = 0; i < 8; i++) {
-                const float *src = slot + (tg + 8 * i) * PS + rg * TR;
-                if constexpr (TR % 4 == 0) {
-#pragma unroll
-                    for (int j = 0; j < TR; j += 4) {
-                        const float4 q4 = *reinterpret_cast<const float4 *>(src + j);
-                        v[i][j] += q4.x;
-                        v[i][j + 1] += q4.y;
-                        v[i][j + 2] += q4.z;
-                        v[i][j + 3] += q4.w;
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < TR; j++) v[i][j] += src[j];
-                }
-            }
-        }
-        ptx::named_barrier(1, NW * 32);
+    if (S == 1) {   // one warp per item: no partial tiles to combine
+        if (has_item) store_tile<T, TR, NRG>(a, sh, v, gi, n0, rg, tg, ks);
+        return;
     }
-    if (!has_item || piece != 0 || ks != 0) return;
-    store_tile<T, TR, NRG>(a, sh, v, gi, n0, rg, tg);
+    // every warp's tile to its slot (slot = warp = item * S + piece), then
+    // the output pass over all items
+    if (has_item) write_slot<TR, NRG, PS>(slots, warp, v, tg, rg, ks);
+    ptx::named_barrier(1, NW * 32);
+    output_pass<T, R, NW, PS>(a, sh, slots, S, g_count, n0, warp, lane);
 }
 
 template <typename T, int TR, int NRG, int CT, int RW, int NW>
 __global__ void __launch_bounds__((NW + 1) * 32, 1)
 k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     using St = Stage<T>;
-    constexpr int R = TR * NRG;
     extern __shared__ unsigned char smem_raw[];
     Shared sh;
     sh.base = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -580,7 +628,6 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     const int64_t n0 = (cluster_id % n_tiles) * TN;
     const int item_first = task * a.G;
     const int g_count = task < a.n_tasks ? min(a.G, a.n_items - item_first) : 0;
-    const int C = CT ? CT : a.C;
     const int nch = a.nchunks;
 
     if (threadIdx.x == 0) {
@@ -590,7 +637,6 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
         }
         ptx::mbar_init(sh.wbar, 1);
         sh.misc[0] = 0;
-        sh.misc[3] = 1;
         ptx::fence_barrier_init();
     }
     // every CTA's barriers exist before any multicast or remote arrive
@@ -682,11 +728,12 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// ring, reused for the epilogue's partial tiles
+// The ring, reused after the main loop for the warps' tile slots (one per
+// consumer warp, or one per item for one-row blocks, up to two per warp).
 size_t region_bytes(bsr_dtype_t dt, int R) {
     const size_t ring = (size_t)NS * (dt == BSR_F32 ? Stage<float>::kBytes : Stage<uint16_t>::kBytes);
-    const int nw = R == 1 ? kXsConsumerWarpsR1 : NCW;
-    const size_t part = (size_t)(nw * 2 / 3) * TN * (R + 4) * 4;   // most tiles of one tree round (S=3)
+    const int nslots = R == 1 ? 2 * kXsConsumerWarpsR1 : NCW;
+    const size_t part = (size_t)TN * xstage_slot_pitch(R, nslots) * 4;
     return (std::max(ring, part) + 1023) & ~size_t(1023);
 }
 

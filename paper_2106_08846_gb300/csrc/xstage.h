@@ -56,6 +56,17 @@ XS_HD inline int xstage_block_ints(int R, int C) { return R == 1 && C == 1 ? 2 :
 XS_HD inline int64_t xstage_record_ints(int64_t len, int64_t nchunks, int bi = 1) {
     return xstage_pad4(bi * len) + xstage_pad4(nchunks + 1);
 }
+// Tile slots, written by the consumer warps after the main loop (in the
+// ring, then free): token-major, [t][slot][r], so that the output pass reads
+// consecutive outputs of one token from consecutive banks. The token pitch
+// (floats) is padded so that eight consecutive tokens of one slot land in
+// distinct 16-byte bank groups (one-row and two-row tiles: distinct banks).
+constexpr int xstage_slot_pitch(int R, int nslot) {
+    const int base = nslot * R;
+    if (R == 1) return base % 2 == 0 ? base + 1 : base;
+    if (R == 2) return (base / 2) % 2 == 0 ? base + 2 : base;
+    return base % 8 == 4 ? base : base + (12 - base % 8) % 8;
+}
 // Byte offset of chunk column kk inside a ring stage, token row 0.
 uint32_t xstage_stage_offset(bsr_dtype_t dt, int kk);
 
