@@ -8,9 +8,14 @@ N(0, 1), bias N(0, 0.02). One step = one bsr_spmm call per shape (8 calls).
 
 Metric: useful GFLOP/s = sum over calls of 2*N*nnz (nnz = stored block
 elements) / device time, inputs resident in HBM, L2 flushed (a 512 MiB write)
-before every timed step and not timed. Per-kernel CUDA events inside the timed
-region give each kernel's average duration; the one with the largest share is
-reported against its roofline. ``e2e`` repeats the step through the C ABI
+before every timed step and not timed. The timed steps carry CUDA events
+only at step boundaries: consecutive launches of a step overlap (each kernel
+starts its prologue while the previous one finishes, see the library's
+programmatic launches), and an event between them would serialise them. A
+second pass over the same steps, inside the same clock-sampled region, puts
+an event pair around every launch to give each kernel's average duration
+(per_shape); the kernel with the largest share is reported against its
+roofline. ``e2e`` repeats the step through the C ABI
 with pinned host X and Y (the library copies in and out on the stream).
 ``cpu_baseline`` times the CPU oracle on the host cores.
 
@@ -323,14 +328,24 @@ def run_ours(args, world, rank, local):
         # hold the stream while the host enqueues every timed launch, so that
         # the events time back-to-back device execution, not host launch gaps
         torch.cuda._sleep(int((enqueue_s * K * 2.0 + 0.05) * clock_mhz * 1e6))
+        # the timed steps: events only at step boundaries, so that nothing
+        # sits between the launches of a step (an event record there would
+        # stop a kernel from starting while the previous one finishes)
         for k in range(K):
             flush.zero_()
             st[k][0].record(stream)
+            step()
+            st[k][1].record(stream)
+        torch.cuda.synchronize()
+        # per-kernel durations: the same steps again with an event pair
+        # around every launch (for per_shape and the roofline)
+        torch.cuda._sleep(int((enqueue_s * K * 2.0 + 0.05) * clock_mhz * 1e6))
+        for k in range(K):
+            flush.zero_()
             for i, (h, b, Y) in enumerate(zip(handles, biases, Ys)):
                 ev[k][i][0].record(stream)
                 bsr.bsr_spmm(h, X, b, Y, N, stream)
                 ev[k][i][1].record(stream)
-            st[k][1].record(stream)
         torch.cuda.synchronize()
     barrier(world)
     step_ms = [a.elapsed_time(b) for a, b in st]

@@ -6,6 +6,8 @@
 
 #include "bsr_internal.h"
 #include "elem.cuh"
+#include "launch.cuh"
+#include "ptx.cuh"
 
 namespace bsr {
 
@@ -17,6 +19,8 @@ k_generic(const Item *__restrict__ items, int n_items, const int32_t *__restrict
           const T *__restrict__ data, const T *__restrict__ X, const float *__restrict__ bias,
           T *__restrict__ Y, float *__restrict__ ws, int64_t N, int64_t K, int64_t M, int R, int C,
           int tn, int64_t n_tiles) {
+    ptx::pdl_launch_dependents();
+    ptx::pdl_wait();   // X, the bias, Y and the workspace may be an earlier kernel's
     const int64_t work = (int64_t)n_items * n_tiles;
     for (int64_t b = blockIdx.x; b < work; b += gridDim.x) {
         const int64_t tile = b / n_items;
@@ -47,6 +51,8 @@ k_generic(const Item *__restrict__ items, int n_items, const int32_t *__restrict
 template <typename T>
 __global__ void k_reduce(const Split *__restrict__ splits, int n_splits, const float *__restrict__ ws,
                          const float *__restrict__ bias, T *__restrict__ Y, int64_t N, int64_t M, int R) {
+    ptx::pdl_launch_dependents();
+    ptx::pdl_wait();   // the partials come from the product kernel just before
     const int64_t total = (int64_t)n_splits * N * R;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
          e += (int64_t)gridDim.x * blockDim.x) {
@@ -72,15 +78,12 @@ cudaError_t launch_generic(const LaunchArgs &a) {
     const int64_t work = (int64_t)n_items * n_tiles;
     const int grid = (int)std::min<int64_t>(work, 1 << 24);
     if (sc.dt == BSR_F32)
-        k_generic<float><<<grid, 256, 0, a.stream>>>(sc.d_items, n_items, sc.d_indices, (const float *)a.data,
-                                                     (const float *)a.X, a.bias, (float *)a.Y, a.ws, a.N,
-                                                     sc.K, sc.M, sc.R, sc.C, tn, n_tiles);
-    else
-        k_generic<uint16_t><<<grid, 256, 0, a.stream>>>(sc.d_items, n_items, sc.d_indices,
-                                                        (const uint16_t *)a.data, (const uint16_t *)a.X,
-                                                        a.bias, (uint16_t *)a.Y, a.ws, a.N, sc.K, sc.M,
-                                                        sc.R, sc.C, tn, n_tiles);
-    return cudaGetLastError();
+        return launch_kernel(k_generic<float>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Item *)sc.d_items,
+                             n_items, (const int32_t *)sc.d_indices, (const float *)a.data, (const float *)a.X,
+                             a.bias, (float *)a.Y, a.ws, a.N, sc.K, sc.M, sc.R, sc.C, tn, n_tiles);
+    return launch_kernel(k_generic<uint16_t>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Item *)sc.d_items,
+                         n_items, (const int32_t *)sc.d_indices, (const uint16_t *)a.data, (const uint16_t *)a.X,
+                         a.bias, (uint16_t *)a.Y, a.ws, a.N, sc.K, sc.M, sc.R, sc.C, tn, n_tiles);
 }
 
 cudaError_t launch_reduce(const LaunchArgs &a) {
@@ -90,12 +93,10 @@ cudaError_t launch_reduce(const LaunchArgs &a) {
     const int64_t total = (int64_t)n_splits * a.N * sc.R;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, 1 << 20));
     if (sc.dt == BSR_F32)
-        k_reduce<float><<<grid, 256, 0, a.stream>>>(sc.d_splits, n_splits, a.ws, a.bias, (float *)a.Y, a.N,
-                                                    sc.M, sc.R);
-    else
-        k_reduce<uint16_t><<<grid, 256, 0, a.stream>>>(sc.d_splits, n_splits, a.ws, a.bias,
-                                                       (uint16_t *)a.Y, a.N, sc.M, sc.R);
-    return cudaGetLastError();
+        return launch_kernel(k_reduce<float>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
+                             n_splits, (const float *)a.ws, a.bias, (float *)a.Y, a.N, sc.M, sc.R);
+    return launch_kernel(k_reduce<uint16_t>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
+                         n_splits, (const float *)a.ws, a.bias, (uint16_t *)a.Y, a.N, sc.M, sc.R);
 }
 
 }  // namespace bsr

@@ -32,6 +32,7 @@
 
 #include "bsr_internal.h"
 #include "elem.cuh"
+#include "launch.cuh"
 #include "ptx.cuh"
 #include "tc.h"
 
@@ -156,6 +157,7 @@ __device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[3
 template <typename T, int R>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
+    ptx::pdl_launch_dependents();
     constexpr bool F32 = sizeof(T) == 4;
     constexpr int NS = TcCfg<T>::NS;
     extern __shared__ unsigned char smem_raw[];
@@ -223,6 +225,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
             const uint32_t rec_bytes = (uint32_t)(pad4(nch + 2) + pad4(n_ent)) * 4;
             ptx::mbar_arrive_expect_tx(rbar, rec_bytes);
             ptx::bulk_load(I_s, trec, rec_bytes, rbar);
+            ptx::pdl_wait();   // X may be an earlier kernel's output
             const unsigned char *wsrc = static_cast<const unsigned char *>(a.wpk);
             int k = 0;          // ring slots used (chunks with work, in order)
             int stalled = -1;   // test hook: the slot left empty
@@ -345,6 +348,7 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
         // ---------------- warps 2..5: fp32 split during the main loop, then
         // the epilogue; TMEM lane quarter = warp % 4
         const int et = threadIdx.x - 64;   // 0..127
+        ptx::pdl_wait();   // the bias, Y and the workspace may be an earlier kernel's
         for (int e = et; e < g_count * R; e += 128) {
             const int g = e / R, r = e - g * R;
             B_s[e] = a.bias ? __ldg(a.bias + (int64_t)itab[6 * g + 0] * R + r) : 0.f;
@@ -575,7 +579,8 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     const int64_t n_tiles = (la.N + TN - 1) / TN;
     const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
     if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-    k_tc<T, R><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
+    const cudaError_t e = launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem, la.stream, 1u, map, a);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -44,6 +44,7 @@
 
 #include "bsr_internal.h"
 #include "elem.cuh"
+#include "launch.cuh"
 #include "ptx.cuh"
 #include "xstage.h"
 
@@ -495,6 +496,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         }
     }
     ptx::named_barrier(1, NW * 32);
+    ptx::pdl_wait();   // the bias, Y and the workspace may be an earlier kernel's
     // the bias, needed only by the output pass (waited for there)
     for (int e = ctid; e < g_count * R; e += NW * 32) {
         const int g = e / R, r = e - g * R;
@@ -618,6 +620,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     sh.W = reinterpret_cast<float *>(sh.base + a.blob_off + a.hdr + a.ib);
     sh.B = reinterpret_cast<float *>(sh.base + a.bias_off);
 
+    ptx::pdl_launch_dependents();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // clusters in tile-fastest order (concurrent clusters spread over tiles);
     // the CTAs of a cluster take consecutive tasks of the same tile
@@ -650,6 +653,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
                 ptx::bulk_load(sh.itab, a.blob + (int64_t)task * a.stride, a.stride, sh.wbar);
             }
             ptx::prefetch_tensormap(&xmap);
+            ptx::pdl_wait();   // X may be an earlier kernel's output
             const int rows = TN / (int)CL;                       // this CTA's slice of every chunk
             const uint16_t mask = (uint16_t)((1u << CL) - 1u);
             int c = 0;
@@ -848,24 +852,8 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-        if (CL == 1) {
-            k_xstage<T, TR, NRG, CT, RW, NW><<<(unsigned)grid, NTHREADS, smem, la.stream>>>(map, a);
-            err = cudaGetLastError();
-            break;
-        }
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3((unsigned)grid);
-        cfg.blockDim = dim3(NTHREADS);
-        cfg.dynamicSmemBytes = smem;
-        cfg.stream = la.stream;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = (unsigned)CL;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        err = cudaLaunchKernelEx(&cfg, k_xstage<T, TR, NRG, CT, RW, NW>, map, a);
+        err = launch_kernel(k_xstage<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem, la.stream,
+                            (unsigned)CL, map, a);
         break;
     }
     return err;
