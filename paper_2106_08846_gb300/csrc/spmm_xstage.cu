@@ -695,7 +695,8 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
 // blobs + vdst[g * n_items + i] (floats; -1: none), blocks in the records'
 // order (perm: position -> stored block), per block W^T widened to fp32
 // with WD copies: [(b*C + c)*R + r]*stride + d <- data[(perm[p0_i + b]*R + r)*C + c]
-// (stride WD, or 2 for 1x1 blocks whose weights sit beside their offsets).
+// (stride WD; 1x1 blocks: stride 2 and one copy, the weight beside its X
+// offset in the record).
 template <typename T>
 __global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ items, const int32_t *__restrict__ perm,
                        const int64_t *__restrict__ vdst, int64_t n_items, float *__restrict__ blobs, int R, int C,
@@ -711,7 +712,8 @@ __global__ void k_pack(const T *__restrict__ data, const Item *__restrict__ item
             const int rc = (int)(e - b * R * C);
             const int c = rc / R, r = rc - c * R;
             const float w = to_f32(data[((int64_t)perm[it.p0 + b] * R + r) * C + c]);
-            for (int k = 0; k < WD; k++) dst[stride * e + k] = w;
+            const int copies = R == 1 && C == 1 ? 1 : WD;
+            for (int k = 0; k < copies; k++) dst[stride * e + k] = w;
         }
     }
 }
