@@ -62,7 +62,8 @@ void make_items(Schedule &sc, int64_t limit, bool drop_empty = false) {
     // cache lines of Y its output pass writes. Inside each group of twice the
     // consumer warps (a task of two rows per warp), the longest row is paired
     // with the shortest, the second longest with the second shortest, and so
-    // on: warp w owns positions 2w and 2w + 1, so its work is about the mean.
+    // on: warp w owns positions 2w and 2w + 1, so its work is about the mean
+    // (in tasks of four rows per warp it owns two such pairs).
     if (sc.R == 1) {
         const size_t grp = 2 * kXsConsumerWarpsR1;
         std::vector<Item> g;

@@ -1,11 +1,11 @@
 // SIMT BSR x dense kernel with X staged through a TMA ring ("xstage").
 //
 // Each CTA owns a tile of TN = 64 tokens and a task of G work items (block
-// rows or pieces of rows, Section 2.2's kept blocks): S = 12/G consumer
-// warps per item for G <= 12, or G/12 whole items per warp for one-row
-// blocks (12 consumer warps and one producer warp). The inner product over
-// the kept blocks is FP32-FMA bound, so the design goal is a high share of
-// packed FMAs among the issued instructions:
+// rows or pieces of rows, Section 2.2's kept blocks), with NW consumer warps
+// and one producer warp: S = NW/G warps per item for G <= NW (NW = 12), or,
+// for one-row blocks (NW = 24), G/NW whole items per warp when G > NW. The
+// inner product over the kept blocks is FP32-FMA bound, so the design goal
+// is a high share of packed FMAs among the issued instructions:
 //
 //  * The CL CTAs of a thread-block cluster share one token tile (different
 //    tasks). X[n0 : n0+64, k0 : k0+128] chunks stream through a 3-stage
@@ -26,10 +26,16 @@
 //    alternate blocks (or, for wide blocks, a quarter or half of each
 //    block's columns). A lane accumulates an 8 x TR tile with packed
 //    fma.rn.f32x2 over pairs of tokens: (x_t, x_t') * (w, w).
-//  * Epilogue: shuffle-reduce the NKS partials, then sum the S warps of an
-//    item by a fixed pairwise tree through shared memory; the item's first
-//    warp adds the bias, converts and stores from registers (or writes an
-//    fp32 partial for rows split across CTAs).
+//  * Epilogue: shuffle-reduce the NKS partials. A warp that owns whole
+//    items stores its tile straight from registers (one item per warp) or
+//    through a shared-memory slot; the S warps of a shared item write their
+//    partial tiles to slots, and one pass over all of the task's outputs sums
+//    them in piece order, adds the bias, converts and stores row segments of
+//    Y (or writes an fp32 partial for rows split across CTAs).
+//  * The kernel is launched with programmatic stream serialisation: it lets
+//    the next kernel start at once, and fetches its blob and sets up its
+//    barriers before it waits for the previous kernel (X, bias and Y are
+//    touched only after that wait).
 //
 // Every wait is bounded by the global timer; a timeout sets the device
 // status word, stops the CTA's pipeline and drains its TMA loads. A cluster
@@ -735,10 +741,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // The ring, reused after the main loop for the warps' tile slots (one per
-// consumer warp, or one per item for one-row blocks, up to two per warp).
+// consumer warp, or one per item for one-row blocks, up to four per warp).
 size_t region_bytes(bsr_dtype_t dt, int R) {
     const size_t ring = (size_t)NS * (dt == BSR_F32 ? Stage<float>::kBytes : Stage<uint16_t>::kBytes);
-    const int nslots = R == 1 ? 2 * kXsConsumerWarpsR1 : NCW;
+    const int nslots = R == 1 ? 4 * kXsConsumerWarpsR1 : NCW;
     const size_t part = (size_t)TN * xstage_slot_pitch(R, nslots) * 4;
     return (std::max(ring, part) + 1023) & ~size_t(1023);
 }
@@ -872,6 +878,7 @@ cudaError_t launch_w(const LaunchArgs &la, const XsPlan &pl, int G) {
         switch (G > NW ? G / NW : 1) {
             case 1: return G <= NW ? launch_t<T, TR, NRG, CT, 1, NW>(la, pl, G) : cudaErrorInvalidConfiguration;
             case 2: return launch_t<T, TR, NRG, CT, 2, NW>(la, pl, G);
+            case 4: return launch_t<T, TR, NRG, CT, 4, NW>(la, pl, G);
         }
         return cudaErrorInvalidConfiguration;
     } else {
@@ -923,7 +930,7 @@ int g_index(int G) {
 }
 
 bool xstage_task_size_ok(int R, int G) {
-    return R == 1 ? (G <= kXsConsumerWarpsR1 ? kXsConsumerWarpsR1 % G == 0 : G == 2 * kXsConsumerWarpsR1)
+    return R == 1 ? (G <= kXsConsumerWarpsR1 ? kXsConsumerWarpsR1 % G == 0 : (G == 2 * kXsConsumerWarpsR1 || G == 4 * kXsConsumerWarpsR1))
                   : G <= kXsConsumerWarps;
 }
 

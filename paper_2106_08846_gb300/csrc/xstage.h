@@ -17,10 +17,10 @@ constexpr int kXsMaxSmem = 232448;     // 227 KB, the per-CTA opt-in limit
 constexpr int kXsWDup = 1;             // copies of each packed block value
 
 // Task sizes G (items per CTA): up to the consumer warps NW, each dividing
-// them (NW/G warps per item); one-row blocks (NW = 24) also G = 48, two
-// items per warp.
-constexpr int kXsTaskSizes = 8;
-constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12, 24, 48};
+// them (NW/G warps per item); one-row blocks (NW = 24) also G = 48 and 96,
+// two or four items per warp.
+constexpr int kXsTaskSizes = 9;
+constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12, 24, 48, 96};
 
 constexpr int kXsItab = 12;   // ints per item in a task's item table
 
