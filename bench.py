@@ -16,7 +16,8 @@ second pass over the same steps, inside the same clock-sampled region, puts
 an event pair around every launch to give each kernel's average duration
 (per_shape); the kernel with the largest share is reported against its
 roofline. ``e2e`` repeats the step through the C ABI
-with pinned host X and Y (the library copies in and out on the stream).
+with pinned host X and Y (the library copies in and out on the call's stream;
+each weight's calls on a stream of their own).
 ``cpu_baseline`` times the CPU oracle on the host cores.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
@@ -235,17 +236,21 @@ def run_reference(args, world, rank):
 
 def run_e2e(bsr, handles, biases, wl, X_np, N, K, stream, world, flops_step):
     """The step through the C ABI with pinned host X and Y: each call copies X
-    in and Y out on the stream (inside the call), so the copies are timed."""
+    in and Y out (inside the call), so the copies are timed. Each weight's
+    calls run on a stream of their own, as a server would issue independent
+    layers' products: one call's copies then overlap another call's kernel
+    (the host link, about 175 GB/s each way here, carries 50 MB per step)."""
     import torch
     Xh = torch.from_numpy(X_np).pin_memory()
     Yh = [torch.empty((N, w.M), dtype=torch.float32).pin_memory() for w in wl.weights]
-    for h, Y in zip(handles, Yh):
-        bsr.bsr_spmm(h, Xh, None, Y, N, stream)       # sizes the staging buffers
+    streams = [torch.cuda.Stream() for _ in handles]
+    for h, Y, st in zip(handles, Yh, streams):
+        bsr.bsr_spmm(h, Xh, None, Y, N, st)       # sizes the staging buffers
     torch.cuda.synchronize()
 
     def e2e_step():
-        for h, b, Y in zip(handles, biases, Yh):
-            bsr.bsr_spmm(h, Xh, b, Y, N, stream)
+        for h, b, Y, st in zip(handles, biases, Yh, streams):
+            bsr.bsr_spmm(h, Xh, b, Y, N, st)
 
     for _ in range(3):
         e2e_step()
@@ -253,8 +258,14 @@ def run_e2e(bsr, handles, biases, wl, X_np, N, K, stream, world, flops_step):
     barrier(world)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    for st in streams:
+        st.wait_event(e0)
     for _ in range(K):
         e2e_step()
+    for st in streams:   # the timed region ends when every stream's last call has finished
+        done = torch.cuda.Event()
+        done.record(st)
+        stream.wait_event(done)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
