@@ -535,7 +535,8 @@ int choose_tasks(const Schedule &sc, int64_t N) {
 }
 
 // Task size for the tcgen05 kernel: the same waves x (overhead + work) model,
-// among the G whose accumulators fit tensor memory and whose shared memory fits.
+// among the G whose accumulators fit tensor memory and whose shared memory
+// fits; a wave is every SM holding as many CTAs as fit it at once.
 int choose_tc_tasks(const Schedule &sc, int64_t N) {
     static const int forced = [] {
         const char *v = getenv("BSR_TC_G");
@@ -553,7 +554,9 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
         const int G = kTcG[gi];
         if (!fits(G)) continue;
         const int64_t ctas = tiles * ((items + G - 1) / G);
-        const double waves = (double)((ctas + sc.sm_count - 1) / sc.sm_count);
+        const int64_t slots = (int64_t)sc.sm_count *
+                              tc_ctas_per_sm(sc.R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt);
+        const double waves = (double)((ctas + slots - 1) / slots);
         const double cost = waves * (kOverheadItems + (double)std::min<int64_t>(G, items));
         if (best_cost < 0 || cost < best_cost) {
             best_cost = cost;

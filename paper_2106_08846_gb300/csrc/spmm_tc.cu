@@ -155,7 +155,7 @@ __device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[3
 }
 
 template <typename T, int R>
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(NTHREADS, sizeof(T) == 4 ? 2 : 1)
 k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
     ptx::pdl_launch_dependents();
     constexpr bool F32 = sizeof(T) == 4;
@@ -607,6 +607,15 @@ size_t tc_smem_bytes(int R, int G, size_t wstage, size_t ibytes, bsr_dtype_t dt)
     const int ns = dt == BSR_F32 ? kTcStagesF32 : kTcStages;
     return ring + ns * ((wstage + 15) & ~size_t(15)) + ((ibytes + 15) & ~size_t(15)) +
            (((size_t)G * R * 4 + 15) & ~size_t(15)) + (3 * ns + 2) * 8 + (4 + 6 * 32) * 4 + 1024;
+}
+
+int tc_ctas_per_sm(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt) {
+    constexpr size_t kSmemPerSm = 233472;   // 228 KB, of which 1 KB is reserved per CTA
+    const size_t per_cta = tc_smem_bytes(R, G, wbytes, ibytes, dt) + 1024;
+    const int by_smem = (int)(kSmemPerSm / per_cta);
+    const int by_tmem = kTcTmemCols / (int)tmem_cols_for(G * R);
+    const int bound = dt == BSR_F32 ? 2 : 1;   // the kernel's __launch_bounds__
+    return std::max(1, std::min(bound, std::min(by_smem, by_tmem)));
 }
 
 size_t tc_task_budget(int R, bsr_dtype_t dt) {

@@ -12,7 +12,8 @@ namespace bsr {
 constexpr int kTcTokens = 128;         // tokens per CTA = MMA M = TMEM lanes
 constexpr int kTcChunk = 64;           // K columns per ring stage (one 128-byte swizzle row of bf16)
 constexpr int kTcStages = 6;           // ring depth (bf16)
-constexpr int kTcStagesF32 = 4;        // ring depth (fp32: each stage has a twin for the low parts)
+constexpr int kTcStagesF32 = 2;        // ring depth (fp32: each stage has a twin for the low parts; two
+                                       // stages let two CTAs share an SM and overlap their stage latencies)
 constexpr int kTcMaxSmem = 232448;     // 227 KB
 constexpr int kTcTmemCols = 512;       // accumulator columns per SM
 constexpr int kTcTaskSizes = 6;
@@ -47,6 +48,9 @@ bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 int tc_g_index(int G);
 size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt);
 size_t tc_task_budget(int R, bsr_dtype_t dt);
+// CTAs of the tensor-core kernel that fit one SM at once (shared memory,
+// tensor memory and the kernel's launch bound), for a task size's footprint.
+int tc_ctas_per_sm(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt);
 // K columns per ring stage: one 128-byte swizzle row (64 bf16 or 32 fp32)
 inline int tc_chunk_cols(bsr_dtype_t dt) { return dt == BSR_F32 ? 32 : 64; }
 // bytes of one block's B operand(s): bf16, or fp32 high and low tf32 parts
