@@ -391,6 +391,15 @@ def run_ours(args, world, rank, local):
             f"{pk.get('sm_max_mhz', 2070.0)} MHz ({pk['source']} max clock)"),
         "hbm_frac": (nbytes[dom] / (kern_ms[dom] * 1e-3) / 1e9) / float(pk["hbm_gbs"]),
     }
+    if w.R == 1 and variant == "xstage":
+        # a one-row block reuses no X value across outputs: every FMA needs one
+        # 4-byte shared-memory load, and shared memory serves 128 bytes per
+        # clock per SM, so such a kernel cannot exceed 32 FMA per clock per SM
+        smem_tflops = props.multi_processor_count * 32 * 2 * float(pk.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+        roofline["smem_ceiling"] = {
+            "peak": smem_tflops, "unit": "TFLOP/s", "frac": achieved / smem_tflops,
+            "source": f"derived: {props.multi_processor_count} SMs x 32 fp32 shared loads/clock x 2 flop x "
+                      f"{pk.get('sm_max_mhz', 2070.0)} MHz (one load per FMA)"}
     per_shape = {f"{wl.weights[i].R}x{wl.weights[i].C}": {
         "us": round(kern_ms[i] * 1e3, 2), "gflops": round(flops[i] / (kern_ms[i] * 1e-3) / 1e9, 1),
         "gbs": round(nbytes[i] / (kern_ms[i] * 1e-3) / 1e9, 1), "variant": scheds[i]["variant"],
