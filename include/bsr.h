@@ -175,6 +175,35 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len);
 bsr_status_t bsr_spmm_noalloc(bsr_handle_t h, const void *X, const float *bias, void *Y, int64_t N,
                               void *stream);
 
+/*
+ * bsr_spmm_batch -- n products that share one input: Y_i = X · W_iᵀ + b_i.
+ *
+ * The paper prunes BERT (Section 2.3), whose self-attention applies several
+ * weights (query, key, value) to the same activations; this entry point takes
+ * such products together. Products whose weights run on the SIMT kernel with the
+ * same kernel configuration (same dtype and block shape, and the same task
+ * layout for the call's N) are fused into one grid -- up to 64 per launch --
+ * so one product's last, partly filled wave overlaps the others' work; every
+ * other product runs after it, in order, on the same stream. Each output is
+ * bit-identical to what bsr_spmm gives for the same arguments.
+ *
+ *   handles[n]  distinct handles, all on one device, one dtype and one K;
+ *               BSR_ERR_INVALID_ARG for a NULL or repeated handle or a device
+ *               or dtype mismatch, BSR_ERR_SHAPE for a K mismatch.
+ *   X           device, [N, K] row-major, 16-byte aligned; read by all.
+ *   biases      NULL (no bias anywhere) or n entries, each NULL or a device
+ *               fp32 [M_i] array (4-byte aligned).
+ *   Ys[n]       device, [N, M_i] row-major, 16-byte aligned; no output may
+ *               overlap X, a bias or another output (BSR_ERR_INVALID_ARG).
+ *   N           tokens; n == 0 or N == 0 is a no-op returning BSR_OK.
+ *   stream      as in bsr_spmm. Host buffers are not accepted (BSR_ERR_INVALID_ARG).
+ *
+ * Asynchronous; like bsr_spmm it may grow a handle's split-row workspace (with
+ * one stream synchronisation) unless bsr_reserve sized it for N beforehand.
+ */
+bsr_status_t bsr_spmm_batch(const bsr_handle_t *handles, int n, const void *X, const float *const *biases,
+                            void *const *Ys, int64_t N, void *stream);
+
 /* bsr_destroy -- release what the handle owns (not the borrowed arrays). NULL is a no-op. */
 void bsr_destroy(bsr_handle_t h);
 

@@ -63,6 +63,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.bsr_spmm.restype = U
         lib.bsr_spmm_noalloc.argtypes = [P, P, P, P, I64, P]
         lib.bsr_spmm_noalloc.restype = U
+        lib.bsr_spmm_batch.argtypes = [ctypes.POINTER(P), ctypes.c_int, P, ctypes.POINTER(P), ctypes.POINTER(P),
+                                       I64, P]
+        lib.bsr_spmm_batch.restype = U
         lib.bsr_check_device_status.argtypes = [P]
         lib.bsr_check_device_status.restype = U
         lib.bsr_get_schedule.argtypes = [P, ctypes.c_char_p, ctypes.c_size_t]
@@ -220,6 +223,33 @@ def bsr_spmm_noalloc(h: Handle, X: torch.Tensor, bias: Optional[torch.Tensor], Y
     if X.shape[-1] != h.K or Y.shape[-1] != h.M or X.shape[0] < N or Y.shape[0] < N:
         raise ValueError("X must be [N, K] and Y [N, M]")
     _check(load().bsr_spmm_noalloc(h.ptr, _ptr(X), _ptr(bias), _ptr(Y), N, _stream(stream)), "bsr_spmm_noalloc")
+
+
+def bsr_spmm_batch(handles, X: torch.Tensor, biases, Ys, N: Optional[int] = None, stream=None) -> None:
+    """Ys[i][N, M_i] = X[N, K] W_i^T + biases[i] for handles sharing X (device
+    tensors only); fused products run as one grid (see include/bsr.h)."""
+    n = len(handles)
+    if len(Ys) != n or (biases is not None and len(biases) != n):
+        raise ValueError("one output (and bias, if given) per handle")
+    if not X.is_contiguous():
+        raise ValueError("X must be contiguous")
+    N = X.shape[0] if N is None else N
+    if n and (X.shape[-1] != handles[0].K or X.shape[0] < N):
+        raise ValueError("X must be [N, K]")   # (a K that differs between handles: BSR_ERR_SHAPE)
+    for h, Y in zip(handles, Ys):
+        if X.dtype != h.dtype or Y.dtype != h.dtype:
+            raise TypeError("X and every Y must have the handles' dtype")
+        if not Y.is_contiguous() or Y.shape[-1] != h.M or Y.shape[0] < N:
+            raise ValueError("each Y must be [N, M] and contiguous")
+    if biases is not None:
+        for b in biases:
+            if b is not None and (b.dtype != torch.float32 or not b.is_contiguous()):
+                raise TypeError("biases must be contiguous float32 tensors")
+    P = ctypes.c_void_p
+    harr = (P * max(n, 1))(*[h.ptr for h in handles])
+    yarr = (P * max(n, 1))(*[_ptr(Y) for Y in Ys])
+    barr = None if biases is None else (P * max(n, 1))(*[_ptr(b) for b in biases])
+    _check(load().bsr_spmm_batch(harr, n, _ptr(X), barr, yarr, N, _stream(stream)), "bsr_spmm_batch")
 
 
 def bsr_check_device_status(h: Handle) -> int:

@@ -364,6 +364,72 @@ bsr_status_t bsr_spmm(bsr_handle_t h, const void *X, const float *bias, void *Y,
     return BSR_OK;
 }
 
+bsr_status_t bsr_spmm_batch(const bsr_handle_t *handles, int n, const void *X, const float *const *biases,
+                            void *const *Ys, int64_t N, void *stream) {
+    if (n < 0 || N < 0) return BSR_ERR_INVALID_ARG;
+    if (n == 0 || N == 0) return BSR_OK;
+    if (!handles || !X || !Ys) return BSR_ERR_INVALID_ARG;
+    for (int i = 0; i < n; i++) {
+        if (!handles[i] || !Ys[i]) return BSR_ERR_INVALID_ARG;
+        for (int j = 0; j < i; j++)
+            if (handles[j] == handles[i]) return BSR_ERR_INVALID_ARG;   // one workspace per handle and call
+    }
+    const Handle *h0 = handles[0];
+    for (int i = 1; i < n; i++)
+        if (handles[i]->device != h0->device || handles[i]->dt != h0->dt) return BSR_ERR_INVALID_ARG;
+    for (int i = 0; i < n; i++)
+        if (handles[i]->K != h0->K) return BSR_ERR_SHAPE;
+    const size_t es = dtype_size(h0->dt);
+    const size_t xbytes = (size_t)N * h0->K * es;
+    if ((uintptr_t)X % 16) return BSR_ERR_ALIGNMENT;
+    for (int i = 0; i < n; i++) {
+        if ((uintptr_t)Ys[i] % 16) return BSR_ERR_ALIGNMENT;
+        if (biases && (uintptr_t)biases[i] % 4) return BSR_ERR_ALIGNMENT;
+    }
+    // no output may overlap X, a bias or another output
+    for (int i = 0; i < n; i++) {
+        const size_t yb = (size_t)N * handles[i]->M * es;
+        if (overlaps(X, xbytes, Ys[i], yb)) return BSR_ERR_INVALID_ARG;
+        for (int j = 0; j < n; j++) {
+            if (biases && biases[j] && overlaps(biases[j], (size_t)handles[j]->M * 4, Ys[i], yb))
+                return BSR_ERR_INVALID_ARG;
+            if (j < i && overlaps(Ys[j], (size_t)N * handles[j]->M * es, Ys[i], yb)) return BSR_ERR_INVALID_ARG;
+        }
+    }
+    DeviceGuard g(h0->device);
+    if (!g.ok) return BSR_ERR_CUDA;
+    if (classify(X, h0->device) != PK_DEVICE) return BSR_ERR_INVALID_ARG;   // device buffers only
+    for (int i = 0; i < n; i++) {
+        if (classify(Ys[i], h0->device) != PK_DEVICE) return BSR_ERR_INVALID_ARG;
+        if (biases && biases[i] && classify(biases[i], h0->device) != PK_DEVICE) return BSR_ERR_INVALID_ARG;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    bool synced = false;
+    for (int i = 0; i < n; i++) {
+        Handle *h = handles[i];
+        if ((size_t)h->sched->n_slots * (size_t)N * h->sched->R * 4 <= h->ws_bytes) continue;
+        if (!synced) {
+            if (cudaStreamSynchronize(s) != cudaSuccess) { cudaGetLastError(); return BSR_ERR_CUDA; }
+            synced = true;
+        }
+        bsr_status_t st = reserve_ws(h, N, false);
+        if (st != BSR_OK) return st;
+    }
+    std::vector<LaunchArgs> as;
+    as.reserve((size_t)n);
+    for (int i = 0; i < n; i++) {
+        Handle *h = handles[i];
+        as.push_back(LaunchArgs{h->sched.get(), h->data_packed ? h->data_packed : h->data, X,
+                                biases ? biases[i] : nullptr, Ys[i], h->ws, h->d_status, N, s, h->wait_ns,
+                                h->stall_chunk});
+    }
+    if (launch_spmm_batch(as.data(), n) != cudaSuccess) {
+        cudaGetLastError();
+        return BSR_ERR_CUDA;
+    }
+    return BSR_OK;
+}
+
 bsr_status_t bsr_check_device_status(bsr_handle_t h) {
     if (!h) return BSR_ERR_INVALID_ARG;
     DeviceGuard g(h->device);

@@ -138,6 +138,11 @@ struct LaunchArgs {
 };
 cudaError_t launch_generic(const LaunchArgs &a);
 cudaError_t launch_xstage(const LaunchArgs &a, int G);
+// Products whose xstage launches can share one grid have equal keys (dtype,
+// block shape class and kernel template at task size G).
+int xstage_fusion_key(const Schedule &sc, int G);
+// n products sharing X (equal fusion keys, same X, N, K and stream) in one grid.
+cudaError_t launch_xstage_batch(const LaunchArgs *las, const int *Gs, int n);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
 cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
                          cudaStream_t s);

@@ -566,6 +566,39 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
     return best;
 }
 
+cudaError_t launch_spmm_batch(const LaunchArgs *as, int n) {
+    std::vector<char> done((size_t)std::max(n, 0), 0);
+    std::vector<LaunchArgs> grp;
+    std::vector<int> gs;
+    for (int i = 0; i < n; i++) {
+        if (done[(size_t)i]) continue;
+        if (as[i].sc->variant == V_XSTAGE) {
+            // every later xstage product with the same kernel template joins this grid
+            const int key = xstage_fusion_key(*as[i].sc, choose_tasks(*as[i].sc, as[i].N));
+            grp.clear();
+            gs.clear();
+            for (int j = i; j < n && (int)grp.size() < kXsBatchMax; j++) {
+                if (done[(size_t)j] || as[j].sc->variant != V_XSTAGE) continue;
+                const int G = choose_tasks(*as[j].sc, as[j].N);
+                if (xstage_fusion_key(*as[j].sc, G) != key) continue;
+                grp.push_back(as[j]);
+                gs.push_back(G);
+                done[(size_t)j] = 1;
+            }
+            cudaError_t e = grp.size() == 1 ? launch_xstage(grp[0], gs[0])
+                                            : launch_xstage_batch(grp.data(), gs.data(), (int)grp.size());
+            if (e != cudaSuccess) return e;
+            for (const LaunchArgs &a : grp)
+                if (!a.sc->splits.empty() && (e = launch_reduce(a)) != cudaSuccess) return e;
+            continue;
+        }
+        done[(size_t)i] = 1;
+        cudaError_t e = launch_spmm(as[i]);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
 cudaError_t launch_spmm(const LaunchArgs &a) {
     cudaError_t e;
     if (a.sc->variant == V_TC)

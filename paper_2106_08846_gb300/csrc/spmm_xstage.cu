@@ -610,9 +610,10 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
     output_pass<T, R, NW, PS>(a, sh, slots, S, g_count, n0, warp, lane);
 }
 
+// One CTA of the product described by `a`; `cta` is the CTA's index within
+// that product's grid (clusters of CL consecutive CTAs).
 template <typename T, int TR, int NRG, int CT, int RW, int NW>
-__global__ void __launch_bounds__((NW + 1) * 32, 1)
-k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
+__device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs &a, unsigned cta) {
     using St = Stage<T>;
     extern __shared__ unsigned char smem_raw[];
     Shared sh;
@@ -632,7 +633,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     // the CTAs of a cluster take consecutive tasks of the same tile
     const uint32_t CL = ptx::cluster_nctarank(), rank = ptx::cluster_ctarank();
     const int64_t n_tiles = (a.N + TN - 1) / TN;
-    const int64_t cluster_id = blockIdx.x / CL;
+    const int64_t cluster_id = cta / CL;
     const int task = (int)(cluster_id / n_tiles) * (int)CL + (int)rank;
     const int64_t n0 = (cluster_id % n_tiles) * TN;
     const int item_first = task * a.G;
@@ -695,6 +696,29 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
         consumer<T, TR, NRG, CT, RW, NW>(a, sh, n0, task, g_count, CL, warp, lane);
     }
     if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
+}
+
+template <typename T, int TR, int NRG, int CT, int RW, int NW>
+__global__ void __launch_bounds__((NW + 1) * 32, 1)
+k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
+    xstage_cta<T, TR, NRG, CT, RW, NW>(xmap, a, blockIdx.x);
+}
+
+// Several products sharing X in one grid (no clusters): product h owns CTAs
+// start[h] .. start[h+1]-1, with its own arguments and shared-memory layout
+// (the launch gives every CTA the largest).
+struct XsBatch {
+    int n;
+    unsigned start[kXsBatchMax + 1];
+    XsArgs args[kXsBatchMax];
+};
+
+template <typename T, int TR, int NRG, int CT, int RW, int NW>
+__global__ void __launch_bounds__((NW + 1) * 32, 1)
+k_xstage_batch(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ XsBatch b) {
+    int h = 0;
+    while (h + 1 < b.n && blockIdx.x >= b.start[h + 1]) h++;
+    xstage_cta<T, TR, NRG, CT, RW, NW>(xmap, b.args[h], blockIdx.x - b.start[h]);
 }
 
 // Block values into the task blobs of every task size: item i's values go to
@@ -792,22 +816,19 @@ int choose_cluster(int n_tasks) {
     return 1;
 }
 
-template <typename T, int TR, int NRG, int CT, int RW, int NW>
-cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
+// Kernel arguments and dynamic shared-memory bytes of one product at task
+// size G (nothing to launch: n_items == 0 or N == 0 leaves smem = 0).
+template <int NW>
+cudaError_t make_args(const LaunchArgs &la, const XsPlan &pl, int G, XsArgs &a, uint32_t &smem) {
     const Schedule &sc = *la.sc;
-    const size_t es = sizeof(T);
     const int gidx = g_index(G);
     const int n_items = (int)sc.items.size();
+    smem = 0;
     if (n_items == 0 || la.N == 0) return cudaSuccess;
-    auto enc = encode_fn();
-    if (!enc) return cudaErrorNotSupported;
-
     if (sc.xs_blob_off[gidx] < 0 || la.data == nullptr) return cudaErrorInvalidConfiguration;
-    XsArgs a;
     a.n_items = n_items;
     a.G = G;
     a.S = G <= NW ? NW / G : 1;
-    constexpr int NTHREADS = (NW + 1) * 32;
     a.n_tasks = (n_items + G - 1) / G;
     a.blob = static_cast<const unsigned char *>(la.data) + sc.xs_blob_off[gidx];
     a.stride = (uint32_t)sc.xs_blob_stride[gidx];
@@ -826,45 +847,95 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
     a.bias_off = a.blob_off + a.stride;
     a.bar_off = a.bias_off + (uint32_t)(((size_t)G * sc.R * 4 + 15) & ~size_t(15));
     a.misc_off = a.bar_off + (2 * NS + 1) * 8;
-    const uint32_t smem = a.misc_off + 4 * 4 + 1024;   // + slack to align the base
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
-    static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
+    smem = a.misc_off + 4 * 4 + 1024;   // + slack to align the base
+    return smem > kXsMaxSmem ? cudaErrorInvalidConfiguration : cudaSuccess;
+}
+
+// The 2-D tensor map of X [N, K] for the ring's boxes (rows per box: TN / CL).
+template <typename T>
+cudaError_t encode_x(const void *X, int64_t N, int64_t K, int CL, CUtensorMap *map) {
+    auto enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    const size_t es = sizeof(T);
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)N};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * es};
+    const cuuint32_t box[2] = {(cuuint32_t)Stage<T>::kBoxCols, (cuuint32_t)(TN / CL)};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                     const_cast<void *>(X), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// Opt a kernel into the large dynamic shared memory once per device.
+template <typename K>
+cudaError_t allow_smem(K kernel, std::atomic<uint64_t> &done) {
     int dev = 0;
     cudaGetDevice(&dev);
     const uint64_t bit = 1ull << (dev & 63);
-    if (!(attr_set.load() & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(k_xstage<T, TR, NRG, CT, RW, NW>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kXsMaxSmem);
-        if (e != cudaSuccess) return e;
-        attr_set.fetch_or(bit);
-    }
-    if (smem > kXsMaxSmem) return cudaErrorInvalidConfiguration;
-    const int64_t n_tiles = (la.N + TN - 1) / TN;
+    if (done.load() & bit) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kXsMaxSmem);
+    if (e == cudaSuccess) done.fetch_or(bit);
+    return e;
+}
 
-    cudaError_t err = cudaErrorInvalidConfiguration;
-    for (int CL = choose_cluster(a.n_tasks); CL >= 1; CL >>= 1) {
-        if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT, RW, NW>), CL, smem, dev,
-                                    NTHREADS))
-            continue;
-        const int64_t n_groups = (a.n_tasks + CL - 1) / CL;
-        const int64_t grid = n_tiles * n_groups * CL;   // cluster-major, tile-fastest
-        if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-        CUtensorMap map;
-        const cuuint64_t dims[2] = {(cuuint64_t)sc.K, (cuuint64_t)la.N};
-        const cuuint64_t strides[1] = {(cuuint64_t)sc.K * es};
-        const cuuint32_t box[2] = {(cuuint32_t)Stage<T>::kBoxCols, (cuuint32_t)(TN / CL)};
-        const cuuint32_t estr[2] = {1, 1};
-        CUresult r = enc(&map, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                         const_cast<void *>(la.X), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-        err = launch_kernel(k_xstage<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem, la.stream,
-                            (unsigned)CL, map, a);
-        break;
+// n products sharing X (same dtype, K, N, block shape and template); n == 1
+// is the plain launch (clusters allowed), n > 1 one fused grid.
+template <typename T, int TR, int NRG, int CT, int RW, int NW>
+cudaError_t launch_t(const LaunchArgs *las, const int *Gs, int n, const XsPlan *const *pls) {
+    constexpr int NTHREADS = (NW + 1) * 32;
+    const int64_t n_tiles = (las[0].N + TN - 1) / TN;
+    if (n == 1) {
+        const LaunchArgs &la = las[0];
+        XsArgs a;
+        uint32_t smem = 0;
+        cudaError_t e = make_args<NW>(la, *pls[0], Gs[0], a, smem);
+        if (e != cudaSuccess || smem == 0) return e;
+        static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
+        if ((e = allow_smem(k_xstage<T, TR, NRG, CT, RW, NW>, attr_set)) != cudaSuccess) return e;
+        int dev = 0;
+        cudaGetDevice(&dev);
+        for (int CL = choose_cluster(a.n_tasks); CL >= 1; CL >>= 1) {
+            if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT, RW, NW>), CL, smem,
+                                        dev, NTHREADS))
+                continue;
+            const int64_t n_groups = (a.n_tasks + CL - 1) / CL;
+            const int64_t grid = n_tiles * n_groups * CL;   // cluster-major, tile-fastest
+            if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
+            CUtensorMap map;
+            if ((e = encode_x<T>(la.X, la.N, la.sc->K, CL, &map)) != cudaSuccess) return e;
+            return launch_kernel(k_xstage<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem,
+                                 la.stream, (unsigned)CL, map, a);
+        }
+        return cudaErrorInvalidConfiguration;
     }
-    return err;
+    if (n > kXsBatchMax) return cudaErrorInvalidValue;
+    XsBatch b;
+    b.n = 0;
+    uint32_t smem_max = 0;
+    int64_t grid = 0;
+    for (int i = 0; i < n; i++) {
+        uint32_t smem = 0;
+        cudaError_t e = make_args<NW>(las[i], *pls[i], Gs[i], b.args[b.n], smem);
+        if (e != cudaSuccess) return e;
+        if (smem == 0) continue;   // nothing to do for this product
+        b.start[b.n] = (unsigned)grid;
+        grid += n_tiles * b.args[b.n].n_tasks;
+        smem_max = std::max(smem_max, smem);
+        b.n++;
+    }
+    if (b.n == 0) return cudaSuccess;
+    if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
+    b.start[b.n] = (unsigned)grid;
+    static std::atomic<uint64_t> attr_set_b{0};
+    cudaError_t e = allow_smem(k_xstage_batch<T, TR, NRG, CT, RW, NW>, attr_set_b);
+    if (e != cudaSuccess) return e;
+    CUtensorMap map;
+    if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, 1, &map)) != cudaSuccess) return e;
+    return launch_kernel(k_xstage_batch<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem_max,
+                         las[0].stream, 1u, map, b);
 }
 
 // One-row blocks: kXsConsumerWarpsR1 consumer warps (their register tiles
@@ -872,36 +943,37 @@ cudaError_t launch_t(const LaunchArgs &la, const XsPlan &pl, int G) {
 // per-FMA loop), each owning G/NW items when G exceeds them. Other blocks:
 // kXsConsumerWarps, G <= NW.
 template <typename T, int TR, int NRG, int CT>
-cudaError_t launch_w(const LaunchArgs &la, const XsPlan &pl, int G) {
+cudaError_t launch_w(const LaunchArgs *las, const int *Gs, int n, const XsPlan *const *pls) {
+    const int G = Gs[0];
     if constexpr (TR == 1 && NRG == 1) {
         constexpr int NW = kXsConsumerWarpsR1;
         switch (G > NW ? G / NW : 1) {
-            case 1: return G <= NW ? launch_t<T, TR, NRG, CT, 1, NW>(la, pl, G) : cudaErrorInvalidConfiguration;
-            case 2: return launch_t<T, TR, NRG, CT, 2, NW>(la, pl, G);
-            case 4: return launch_t<T, TR, NRG, CT, 4, NW>(la, pl, G);
+            case 1: return G <= NW ? launch_t<T, TR, NRG, CT, 1, NW>(las, Gs, n, pls) : cudaErrorInvalidConfiguration;
+            case 2: return launch_t<T, TR, NRG, CT, 2, NW>(las, Gs, n, pls);
+            case 4: return launch_t<T, TR, NRG, CT, 4, NW>(las, Gs, n, pls);
         }
         return cudaErrorInvalidConfiguration;
     } else {
         if (G > NCW) return cudaErrorInvalidConfiguration;
-        return launch_t<T, TR, NRG, CT, 1, NCW>(la, pl, G);
+        return launch_t<T, TR, NRG, CT, 1, NCW>(las, Gs, n, pls);
     }
 }
 
 template <typename T, int TR, int NRG>
-cudaError_t launch_c(const LaunchArgs &la, const XsPlan &pl, int G) {
-    if (la.sc->C == 1) return launch_w<T, TR, NRG, 1>(la, pl, G);
-    return launch_w<T, TR, NRG, 0>(la, pl, G);
+cudaError_t launch_c(const LaunchArgs *las, const int *Gs, int n, const XsPlan *const *pls) {
+    if (las[0].sc->C == 1) return launch_w<T, TR, NRG, 1>(las, Gs, n, pls);
+    return launch_w<T, TR, NRG, 0>(las, Gs, n, pls);
 }
 
 template <typename T>
-cudaError_t launch_r(const LaunchArgs &la, const XsPlan &pl, int G) {
-    switch (la.sc->R) {
-        case 1: return launch_c<T, 1, 1>(la, pl, G);
-        case 2: return launch_c<T, 2, 1>(la, pl, G);
-        case 4: return launch_c<T, 4, 1>(la, pl, G);
-        case 8: return launch_c<T, 8, 1>(la, pl, G);
-        case 16: return launch_c<T, 8, 2>(la, pl, G);
-        case 32: return launch_c<T, 8, 4>(la, pl, G);
+cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n, const XsPlan *const *pls) {
+    switch (las[0].sc->R) {
+        case 1: return launch_c<T, 1, 1>(las, Gs, n, pls);
+        case 2: return launch_c<T, 2, 1>(las, Gs, n, pls);
+        case 4: return launch_c<T, 4, 1>(las, Gs, n, pls);
+        case 8: return launch_c<T, 8, 1>(las, Gs, n, pls);
+        case 16: return launch_c<T, 8, 2>(las, Gs, n, pls);
+        case 32: return launch_c<T, 8, 4>(las, Gs, n, pls);
     }
     return cudaErrorNotSupported;
 }
@@ -954,9 +1026,23 @@ cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items
 }
 
 cudaError_t launch_xstage(const LaunchArgs &la, int G) {
-    const XsPlan &pl = la.sc->xs;
-    if (la.sc->dt == BSR_F32) return launch_r<float>(la, pl, G);
-    return launch_r<uint16_t>(la, pl, G);
+    const XsPlan *pl = &la.sc->xs;
+    if (la.sc->dt == BSR_F32) return launch_r<float>(&la, &G, 1, &pl);
+    return launch_r<uint16_t>(&la, &G, 1, &pl);
+}
+
+int xstage_fusion_key(const Schedule &sc, int G) {
+    const int rw = sc.R == 1 && G > kXsConsumerWarpsR1 ? G / kXsConsumerWarpsR1 : 1;
+    return (((int)sc.dt * 64 + sc.R) * 2 + (sc.C == 1 ? 1 : 0)) * 8 + rw;
+}
+
+cudaError_t launch_xstage_batch(const LaunchArgs *las, const int *Gs, int n) {
+    if (n <= 0) return cudaSuccess;
+    if (n > kXsBatchMax) return cudaErrorInvalidValue;
+    const XsPlan *pls[kXsBatchMax];
+    for (int i = 0; i < n; i++) pls[i] = &las[i].sc->xs;
+    if (las[0].sc->dt == BSR_F32) return launch_r<float>(las, Gs, n, pls);
+    return launch_r<uint16_t>(las, Gs, n, pls);
 }
 
 }  // namespace bsr

@@ -15,6 +15,7 @@ constexpr int kXsConsumerWarps = 12;   // + 1 producer warp: 16 warps of registe
 constexpr int kXsConsumerWarpsR1 = 24; // one-row blocks (small tiles): + 1 producer warp, 80 registers a thread
 constexpr int kXsMaxSmem = 232448;     // 227 KB, the per-CTA opt-in limit
 constexpr int kXsWDup = 1;             // copies of each packed block value
+constexpr int kXsBatchMax = 64;        // products in one fused launch (bsr_spmm_batch)
 
 // Task sizes G (items per CTA): up to the consumer warps NW, each dividing
 // them (NW/G warps per item); one-row blocks (NW = 24) also G = 48 and 96,
