@@ -1,28 +1,37 @@
-// tcgen05 tensor-core BSR x dense kernel for bf16 blocks whose both sides are
-// multiples of 16 ("tc"): every kept block is a dense contraction, so each
-// block of a block row becomes C/16 tcgen05.mma instructions of shape
-// M = 128 tokens, N = R outputs, K = 16, accumulated in fp32 in tensor memory.
+// tcgen05 tensor-core BSR x dense kernel ("tc"): bf16 blocks whose both sides
+// are multiples of 16 (and narrow bf16 blocks re-blocked at create time into
+// zero-filled R x 64 tiles), and fp32 blocks of 32 or more rows as 3xTF32.
+// Every kept block is a dense contraction: C/16 (bf16) or 3 C/8 (fp32)
+// tcgen05.mma instructions of shape M = 128 tokens, N = R outputs,
+// accumulated in fp32 in tensor memory.
 //
-//   warp 0 (one thread)  producer: bulk copies of the task's block values
+//   warp 0 (one thread)  producer: the task's work list by one bulk copy,
+//                         then per K chunk that holds any of the task's
+//                         blocks the X chunk [128 tokens x 128 bytes] by 2-D
+//                         TMA (128-byte swizzle) and, beside it in the same
+//                         stage, the task's block values for that chunk
 //                         (repacked at create time into the MMA's K-major
-//                         core-matrix layout) and item records, then X chunks
-//                         [128 tokens x 64 columns] by 2-D TMA (128-byte
-//                         swizzle) through a 6-stage ring.
+//                         layout, in task-chunk order); chunks without blocks
+//                         are neither loaded nor visited.
 //   warp 1 (one thread)  owns the tensor memory (G * R fp32 columns, one
 //                         block row per R columns) and issues the MMAs from
-//                         the task's work list (built on the host): per K
-//                         chunk, one entry per block of any of the task's
-//                         items in it. Chunks without entries are neither
-//                         loaded nor visited. A tcgen05.commit per chunk
-//                         releases the stage once its MMAs completed.
-//   warps 2..5           epilogue: after the last commit, each reads its 32
-//                         TMEM lanes (tokens), adds the bias, converts to
-//                         bf16 and stores Y (or an fp32 partial for a split
-//                         row).
+//                         the work list (per chunk, one packed entry per
+//                         block: column offset, item, first-block flag); a
+//                         tcgen05.commit per chunk releases the stage.
+//   warps 2..5           fp32: split every landed X stage into tf32 high and
+//                         low parts (low into a twin buffer) for the issuer's
+//                         high x high + high x low + low x high; then the
+//                         epilogue: each reads its 32 TMEM lanes (tokens),
+//                         adds the bias, converts and stores Y (or an fp32
+//                         partial for a split row).
 //
-// Every wait is bounded by the global timer; a timeout sets the device status
-// word, stops issuing, lets the issued copies and MMAs finish, frees the
-// tensor memory and returns.
+// bf16 uses a 6-stage ring, one CTA per SM; fp32 a 2-stage ring (plus the low
+// twins) so that two CTAs share an SM and overlap their stage round trips.
+// Launched with programmatic stream serialisation: set-up and the work list
+// come before the wait for the previous kernel; X, bias, Y after it. Every
+// wait is bounded by the global timer; a timeout sets the device status word,
+// stops issuing, lets the issued copies and MMAs finish, frees the tensor
+// memory and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -42,7 +51,6 @@ namespace {
 
 constexpr int TN = kTcTokens;
 constexpr uint32_t kStageBytes = TN * 128;   // 16 KB: 128 token rows of 128 bytes (64 bf16 or 32 fp32 columns)
-constexpr int kMaxStages = kTcStages;
 // Per element type: K columns per stage and ring depth (fp32 stages come
 // with a second buffer holding the low parts of the split operand).
 template <typename T>
@@ -123,19 +131,6 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// 32 lanes x 16 columns of fp32 from tensor memory.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
-    uint32_t r[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int j = 0; j < 16; j++) v[j] = __uint_as_float(r[j]);
-}
 
 __device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(status, DEV_OK, code); }
 __device__ __forceinline__ bool aborted(const int *flag) { return *reinterpret_cast<const volatile int *>(flag) != 0; }
@@ -617,13 +612,6 @@ int tc_ctas_per_sm(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt) {
     const int bound = dt == BSR_F32 ? 2 : 1;   // the kernel's __launch_bounds__
     return std::max(1, std::min(bound, std::min(by_smem, by_tmem)));
 }
-
-size_t tc_task_budget(int R, bsr_dtype_t dt) {
-    const size_t fixed = tc_smem_bytes(R, 32, 0, 0, dt) + 64;
-    return fixed >= (size_t)kTcMaxSmem ? 0 : (size_t)kTcMaxSmem - fixed;
-}
-
-uint32_t tc_block_offset(int kk) { return (uint32_t)kk * 2; }
 
 cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
                          cudaStream_t s) {

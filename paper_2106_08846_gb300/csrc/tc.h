@@ -47,7 +47,6 @@ inline int64_t tc_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 int tc_g_index(int G);
 size_t tc_smem_bytes(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt);
-size_t tc_task_budget(int R, bsr_dtype_t dt);
 // CTAs of the tensor-core kernel that fit one SM at once (shared memory,
 // tensor memory and the kernel's launch bound), for a task size's footprint.
 int tc_ctas_per_sm(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt);
