@@ -180,12 +180,13 @@ bsr_status_t bsr_spmm_noalloc(bsr_handle_t h, const void *X, const float *bias, 
  *
  * The paper prunes BERT (Section 2.3), whose self-attention applies several
  * weights (query, key, value) to the same activations; this entry point takes
- * such products together. Products whose weights run on the SIMT kernel with the
- * same kernel configuration (same dtype and block shape, and the same task
- * layout for the call's N) are fused into one grid -- up to 64 per launch --
- * so one product's last, partly filled wave overlaps the others' work; every
- * other product runs after it, in order, on the same stream. Each output is
- * bit-identical to what bsr_spmm gives for the same arguments.
+ * such products together. Products whose weights run on the same kernel
+ * configuration -- the SIMT kernel with the same dtype, block shape and task
+ * layout for the call's N, or the tensor-core kernel with the same dtype and
+ * block height -- are fused into one grid, up to 64 per launch, so one
+ * product's last, partly filled wave overlaps the others' work; products on
+ * the generic kernel run one after another on the same stream. Each output
+ * is bit-identical to what bsr_spmm gives for the same arguments.
  *
  *   handles[n]  distinct handles, all on one device, one dtype and one K;
  *               BSR_ERR_INVALID_ARG for a NULL or repeated handle or a device

@@ -144,6 +144,10 @@ int xstage_fusion_key(const Schedule &sc, int G);
 // n products sharing X (equal fusion keys, same X, N, K and stream) in one grid.
 cudaError_t launch_xstage_batch(const LaunchArgs *las, const int *Gs, int n);
 cudaError_t launch_tc(const LaunchArgs &a, int G);
+// Products whose tensor-core launches can share one grid have equal keys.
+int tc_fusion_key(const Schedule &sc);
+// n products sharing X (equal keys, same X, N, K and stream) in one grid.
+cudaError_t launch_tc_batch(const LaunchArgs *las, const int *Gs, int n);
 cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
                          cudaStream_t s);
 cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t nnzb, int R, int C, uint16_t *tiles,

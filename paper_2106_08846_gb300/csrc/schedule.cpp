@@ -567,34 +567,52 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
 }
 
 cudaError_t launch_spmm_batch(const LaunchArgs *as, int n) {
+    // a product's fusion class: its kernel family and the key within it
+    // (-1: runs alone), and its task size for this call
+    auto fusion = [](const LaunchArgs &a, int *G) {
+        if (a.sc->variant == V_XSTAGE) {
+            *G = choose_tasks(*a.sc, a.N);
+            return 2 * xstage_fusion_key(*a.sc, *G);
+        }
+        if (a.sc->variant == V_TC) {
+            *G = choose_tc_tasks(*a.sc, a.N);
+            return 2 * tc_fusion_key(*a.sc) + 1;
+        }
+        *G = 0;
+        return -1;
+    };
     std::vector<char> done((size_t)std::max(n, 0), 0);
     std::vector<LaunchArgs> grp;
     std::vector<int> gs;
     for (int i = 0; i < n; i++) {
         if (done[(size_t)i]) continue;
-        if (as[i].sc->variant == V_XSTAGE) {
-            // every later xstage product with the same kernel template joins this grid
-            const int key = xstage_fusion_key(*as[i].sc, choose_tasks(*as[i].sc, as[i].N));
-            grp.clear();
-            gs.clear();
-            for (int j = i; j < n && (int)grp.size() < kXsBatchMax; j++) {
-                if (done[(size_t)j] || as[j].sc->variant != V_XSTAGE) continue;
-                const int G = choose_tasks(*as[j].sc, as[j].N);
-                if (xstage_fusion_key(*as[j].sc, G) != key) continue;
-                grp.push_back(as[j]);
-                gs.push_back(G);
-                done[(size_t)j] = 1;
-            }
-            cudaError_t e = grp.size() == 1 ? launch_xstage(grp[0], gs[0])
-                                            : launch_xstage_batch(grp.data(), gs.data(), (int)grp.size());
+        int G = 0;
+        const int key = fusion(as[i], &G);
+        if (key < 0) {
+            done[(size_t)i] = 1;
+            cudaError_t e = launch_spmm(as[i]);
             if (e != cudaSuccess) return e;
-            for (const LaunchArgs &a : grp)
-                if (!a.sc->splits.empty() && (e = launch_reduce(a)) != cudaSuccess) return e;
             continue;
         }
-        done[(size_t)i] = 1;
-        cudaError_t e = launch_spmm(as[i]);
+        // every later product of the same class joins this grid
+        const bool tc = as[i].sc->variant == V_TC;
+        const int cap = tc ? kTcBatchMax : kXsBatchMax;
+        grp.clear();
+        gs.clear();
+        for (int j = i; j < n && (int)grp.size() < cap; j++) {
+            if (done[(size_t)j]) continue;
+            int Gj = 0;
+            if (fusion(as[j], &Gj) != key) continue;
+            grp.push_back(as[j]);
+            gs.push_back(Gj);
+            done[(size_t)j] = 1;
+        }
+        const int m = (int)grp.size();
+        cudaError_t e = tc ? (m == 1 ? launch_tc(grp[0], gs[0]) : launch_tc_batch(grp.data(), gs.data(), m))
+                           : (m == 1 ? launch_xstage(grp[0], gs[0]) : launch_xstage_batch(grp.data(), gs.data(), m));
         if (e != cudaSuccess) return e;
+        for (const LaunchArgs &a : grp)
+            if (!a.sc->splits.empty() && (e = launch_reduce(a)) != cudaSuccess) return e;
     }
     return cudaSuccess;
 }

@@ -16,9 +16,9 @@ bsr_status_t pack_data(Handle &h);
 // Launches every kernel of one bsr_spmm call on a.stream.
 cudaError_t launch_spmm(const LaunchArgs &a);
 
-// Launches n products that share X, N and the stream: xstage products whose
-// kernels share a template run as one grid (up to kXsBatchMax at a time), the
-// others one after another.
+// Launches n products that share X, N and the stream: products whose kernels
+// share a template (xstage, or tensor-core of one dtype and R) run as one
+// grid, up to 64 at a time; generic-kernel products one after another.
 cudaError_t launch_spmm_batch(const LaunchArgs *as, int n);
 
 }  // namespace bsr

@@ -149,9 +149,10 @@ __device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[3
         : "r"(taddr));
 }
 
+// One CTA of the product described by `a`; `cta` is its index in that
+// product's grid (tile-fastest).
 template <typename T, int R>
-__global__ void __launch_bounds__(NTHREADS, sizeof(T) == 4 ? 2 : 1)
-k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
+__device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a, unsigned cta) {
     ptx::pdl_launch_dependents();
     constexpr bool F32 = sizeof(T) == 4;
     constexpr int NS = TcCfg<T>::NS;
@@ -171,8 +172,8 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t n_tiles = (a.N + TN - 1) / TN;
-    const int task = (int)(blockIdx.x / n_tiles);
-    const int64_t n0 = (int64_t)(blockIdx.x % n_tiles) * TN;
+    const int task = (int)(cta / n_tiles);
+    const int64_t n0 = (int64_t)(cta % n_tiles) * TN;
     const int item_first = task * a.G;
     const int g_count = min(a.G, a.n_items - item_first);
     const int C = a.C, nch = a.nchunks;
@@ -442,6 +443,29 @@ k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
     }
 }
 
+template <typename T, int R>
+__global__ void __launch_bounds__(NTHREADS, sizeof(T) == 4 ? 2 : 1)
+k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
+    tc_cta<T, R>(xmap, a, blockIdx.x);
+}
+
+// Several products sharing X in one grid: product h owns CTAs start[h] ..
+// start[h+1]-1, with its own arguments (the launch gives every CTA the
+// largest shared memory of the group).
+struct TcBatch {
+    int n;
+    unsigned start[kTcBatchMax + 1];
+    TcArgs args[kTcBatchMax];
+};
+
+template <typename T, int R>
+__global__ void __launch_bounds__(NTHREADS, sizeof(T) == 4 ? 2 : 1)
+k_tc_batch(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ TcBatch b) {
+    int h = 0;
+    while (h + 1 < b.n && blockIdx.x >= b.start[h + 1]) h++;
+    tc_cta<T, R>(xmap, b.args[h], blockIdx.x - b.start[h]);
+}
+
 // Block values into the MMA's B operand layout (K-major, no swizzle): for each
 // K-slice of 16 columns, 8-row x 16-byte core matrices, 128 bytes apart along
 // K and 256 bytes apart along the rows.
@@ -514,16 +538,16 @@ uint32_t tmem_cols_for(int cols) {
     return n;
 }
 
+// Kernel arguments and dynamic shared-memory bytes of one product at task
+// size G (nothing to launch: smem = 0).
 template <typename T, int R>
-cudaError_t launch_r(const LaunchArgs &la, int G) {
+cudaError_t make_tc_args(const LaunchArgs &la, int G, TcArgs &a, uint32_t &smem) {
     constexpr int NS = TcCfg<T>::NS, KC = TcCfg<T>::KC;
     const Schedule &sc = *la.sc;
     const int n_items = (int)sc.items.size();
+    smem = 0;
     if (n_items == 0 || la.N == 0) return cudaSuccess;
-    auto enc = encode_fn();
-    if (!enc) return cudaErrorNotSupported;
     const int gidx = tc_g_index(G);
-    TcArgs a;
     a.items = sc.d_items;
     a.n_items = n_items;
     a.G = G;
@@ -550,33 +574,79 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.tmem_cols = tmem_cols_for(G * R);
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
-    const uint32_t smem = a.misc_off + (4 + 6 * 32) * 4 + 1024;
+    smem = a.misc_off + (4 + 6 * 32) * 4 + 1024;
     if (smem > (uint32_t)kTcMaxSmem || G * R > kTcTmemCols) return cudaErrorInvalidConfiguration;
-    static std::atomic<uint64_t> attr_set{0};
+    return cudaSuccess;
+}
+
+template <typename K>
+cudaError_t allow_smem(K kernel, std::atomic<uint64_t> &done) {
     int dev = 0;
     cudaGetDevice(&dev);
     const uint64_t bit = 1ull << (dev & 63);
-    if (!(attr_set.load() & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(k_tc<T, R>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem);
-        if (e != cudaSuccess) return e;
-        attr_set.fetch_or(bit);
-    }
-    CUtensorMap map;
-    const cuuint64_t dims[2] = {(cuuint64_t)sc.K, (cuuint64_t)la.N};
-    const cuuint64_t strides[1] = {(cuuint64_t)sc.K * sizeof(T)};
-    const cuuint32_t box[2] = {(cuuint32_t)KC, (cuuint32_t)TN};
+    if (done.load() & bit) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem);
+    if (e == cudaSuccess) done.fetch_or(bit);
+    return e;
+}
+
+template <typename T>
+cudaError_t encode_x(const void *X, int64_t N, int64_t K, CUtensorMap *map) {
+    auto enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)N};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * sizeof(T)};
+    const cuuint32_t box[2] = {(cuuint32_t)TcCfg<T>::KC, (cuuint32_t)TN};
     const cuuint32_t estr[2] = {1, 1};
-    if (enc(&map, sizeof(T) == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-            const_cast<void *>(la.X), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    if (enc(map, sizeof(T) == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+            const_cast<void *>(X), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+        CUDA_SUCCESS)
         return cudaErrorInvalidValue;
-    const int64_t n_tiles = (la.N + TN - 1) / TN;
-    const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
+    return cudaSuccess;
+}
+
+// n products sharing X (same dtype, R, K, N and stream): n == 1 the plain
+// launch, n > 1 one fused grid.
+template <typename T, int R>
+cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n) {
+    const int64_t n_tiles = (las[0].N + TN - 1) / TN;
+    CUtensorMap map;
+    if (n == 1) {
+        TcArgs a;
+        uint32_t smem = 0;
+        cudaError_t e = make_tc_args<T, R>(las[0], Gs[0], a, smem);
+        if (e != cudaSuccess || smem == 0) return e;
+        static std::atomic<uint64_t> attr_set{0};
+        if ((e = allow_smem(k_tc<T, R>, attr_set)) != cudaSuccess) return e;
+        if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
+        const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
+        if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
+        return launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem, las[0].stream, 1u, map, a);
+    }
+    if (n > kTcBatchMax) return cudaErrorInvalidValue;
+    TcBatch b;
+    b.n = 0;
+    uint32_t smem_max = 0;
+    int64_t grid = 0;
+    for (int i = 0; i < n; i++) {
+        uint32_t smem = 0;
+        cudaError_t e = make_tc_args<T, R>(las[i], Gs[i], b.args[b.n], smem);
+        if (e != cudaSuccess) return e;
+        if (smem == 0) continue;
+        b.start[b.n] = (unsigned)grid;
+        grid += n_tiles * b.args[b.n].n_tasks;
+        smem_max = std::max(smem_max, smem);
+        b.n++;
+    }
+    if (b.n == 0) return cudaSuccess;
     if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-    const cudaError_t e = launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem, la.stream, 1u, map, a);
+    b.start[b.n] = (unsigned)grid;
+    static std::atomic<uint64_t> attr_set_b{0};
+    cudaError_t e = allow_smem(k_tc_batch<T, R>, attr_set_b);
     if (e != cudaSuccess) return e;
-    return cudaGetLastError();
+    if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
+    return launch_kernel(k_tc_batch<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem_max, las[0].stream, 1u, map, b);
 }
 
 }  // namespace
@@ -635,18 +705,26 @@ cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t n
 }
 
 template <typename T>
-cudaError_t launch_tc_t(const LaunchArgs &la, int G) {
-    switch (la.sc->R) {
-        case 16: return launch_r<T, 16>(la, G);
-        case 32: return launch_r<T, 32>(la, G);
-        case 64: return launch_r<T, 64>(la, G);
-        case 128: return launch_r<T, 128>(la, G);
+cudaError_t launch_tc_t(const LaunchArgs *las, const int *Gs, int n) {
+    switch (las[0].sc->R) {
+        case 16: return launch_r<T, 16>(las, Gs, n);
+        case 32: return launch_r<T, 32>(las, Gs, n);
+        case 64: return launch_r<T, 64>(las, Gs, n);
+        case 128: return launch_r<T, 128>(las, Gs, n);
     }
     return cudaErrorNotSupported;
 }
 
 cudaError_t launch_tc(const LaunchArgs &la, int G) {
-    return la.sc->dt == BSR_F32 ? launch_tc_t<float>(la, G) : launch_tc_t<uint16_t>(la, G);
+    return la.sc->dt == BSR_F32 ? launch_tc_t<float>(&la, &G, 1) : launch_tc_t<uint16_t>(&la, &G, 1);
+}
+
+int tc_fusion_key(const Schedule &sc) { return (int)sc.dt * 1024 + sc.R; }
+
+cudaError_t launch_tc_batch(const LaunchArgs *las, const int *Gs, int n) {
+    if (n <= 0) return cudaSuccess;
+    if (n > kTcBatchMax) return cudaErrorInvalidValue;
+    return las[0].sc->dt == BSR_F32 ? launch_tc_t<float>(las, Gs, n) : launch_tc_t<uint16_t>(las, Gs, n);
 }
 
 }  // namespace bsr

@@ -15,6 +15,7 @@ constexpr int kTcStages = 6;           // ring depth (bf16)
 constexpr int kTcStagesF32 = 2;        // ring depth (fp32: each stage has a twin for the low parts; two
                                        // stages let two CTAs share an SM and overlap their stage latencies)
 constexpr int kTcMaxSmem = 232448;     // 227 KB
+constexpr int kTcBatchMax = 64;        // products in one fused launch (bsr_spmm_batch)
 constexpr int kTcTmemCols = 512;       // accumulator columns per SM
 constexpr int kTcTaskSizes = 6;
 constexpr int kTcG[kTcTaskSizes] = {1, 2, 4, 8, 16, 32};

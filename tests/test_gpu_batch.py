@@ -60,35 +60,39 @@ def _run_both(ws, N, dtype, seed, with_bias=True):
     return hs, X, [to_host(y) for y in Yb], [to_host(y) for y in Ys]
 
 
-@pytest.mark.parametrize("R,C,dtype", [(32, 1, "f32"), (1, 1, "f32"), (16, 16, "f32"), (4, 4, "f32"),
-                                       (1, 1, "bf16"), (8, 1, "bf16")])
-def test_batch_matches_single_calls_bitwise_and_oracle(R, C, dtype):
+@pytest.mark.parametrize("R,C,dtype,kind", [(32, 1, "f32", "xstage"), (1, 1, "f32", "xstage"),
+                                            (16, 16, "f32", "xstage"), (4, 4, "f32", "xstage"),
+                                            (1, 1, "bf16", "xstage"), (8, 1, "bf16", "xstage"),
+                                            (16, 16, "bf16", "tcgen05"), (32, 32, "bf16", "tcgen05"),
+                                            (32, 32, "f32", "tcgen05")])
+def test_batch_matches_single_calls_bitwise_and_oracle(R, C, dtype, kind):
     """Three weights of one shape (a query/key/value triple) at different
     sparsities: one fused grid, outputs equal to separate calls bit for bit."""
     N = 200
     ws = [_weight(1500 + 10 * i + R + C, 512, 384, R, C, dtype, d) for i, d in enumerate((0.5, 0.2, 0.05))]
     hs, X, Yb, Ys = _run_both(ws, N, dtype, 1599)
-    assert all(h.schedule()["variant"] == "xstage" for h in hs)
+    assert all(h.schedule()["variant"] == kind for h in hs)
     for w, yb, ys in zip(ws, Yb, Ys):
         assert np.array_equal(yb.view(np.uint8), ys.view(np.uint8))
         check_product(yb, oracle.bsr_from_dense(w.W, w.R, w.C), X, w.bias, w.M)
 
 
 def test_batch_mixed_kernels_split_rows_and_no_bias():
-    """Mixed shapes and kernels in one call (fused groups, tensor-core and
-    generic products in order), a weight with split rows (workspace and reduce
-    pass), different M per weight, no biases."""
+    """Mixed shapes and kernels in one call (a fused xstage group, a fused
+    tensor-core group, a generic product), a weight with split rows (workspace
+    and reduce pass after the fused grid), different M per weight, no biases."""
     N = 333
     ws = [
         _weight(1601, 256, 512, 32, 1, "f32", 0.2),
-        _weight(1602, 512, 512, 32, 32, "f32", 0.3),                 # tensor cores
-        _weight(1603, 384, 512, 32, 1, "f32", 0.05, long_rows=(2, 5)),  # split rows
-        _weight(1604, 255, 512, 3, 2, "f32", 0.2),                   # generic kernel
+        _weight(1602, 512, 512, 32, 32, "f32", 0.3),                     # tensor cores
+        _weight(1603, 384, 512, 32, 1, "f32", 0.05, long_rows=(2, 5)),   # split rows
+        _weight(1604, 255, 512, 3, 2, "f32", 0.2),                       # generic kernel
         _weight(1605, 768, 512, 32, 1, "f32", 0.1),
+        _weight(1606, 256, 512, 32, 32, "f32", 0.05, long_rows=(1,)),    # tensor cores, one long row
     ]
-    hs, X, Yb, Ys = _run_both(ws, N, "f32", 1606, with_bias=False)
+    hs, X, Yb, Ys = _run_both(ws, N, "f32", 1607, with_bias=False)
     kinds = [h.schedule()["variant"] for h in hs]
-    assert kinds == ["xstage", "tcgen05", "xstage", "generic", "xstage"]
+    assert kinds == ["xstage", "tcgen05", "xstage", "generic", "xstage", "tcgen05"]
     assert hs[2].schedule()["split_rows"] >= 1
     for w, yb, ys in zip(ws, Yb, Ys):
         assert np.array_equal(yb, ys)
