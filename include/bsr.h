@@ -134,8 +134,9 @@ bsr_status_t bsr_check_device_status(bsr_handle_t h);
 
 /*
  * bsr_get_schedule -- a text description of the handle's schedule: kernel
- * variant, execution block width (exec_C: 64 where narrow bf16 blocks run on
- * the tensor cores as zero-filled R x 64 tiles), tile sizes, work items, split
+ * variant, execution block height and width (exec_R x exec_C: max(R, 16) x 64
+ * where small or narrow bf16 blocks run on the tensor cores as zero-filled
+ * tiles), tile sizes, work items, split
  * rows, launches per call and the schedule-cache statistics, as "key=value"
  * lines. Writes at most len bytes
  * including the terminating NUL into buf (truncating). Returns

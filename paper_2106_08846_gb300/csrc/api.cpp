@@ -298,7 +298,7 @@ bsr_status_t bsr_create(const int32_t *indptr, const int32_t *indices, const voi
 static bsr_status_t reserve_ws(Handle *h, int64_t N, bool host_io) {
     const Schedule &sc = *h->sched;
     size_t es = dtype_size(h->dt);
-    bsr_status_t st = grow((void **)&h->ws, &h->ws_bytes, (size_t)sc.n_slots * (size_t)N * sc.R * 4);
+    bsr_status_t st = grow((void **)&h->ws, &h->ws_bytes, (size_t)sc.n_slots * (size_t)N * sc.ex_R * 4);
     if (st == BSR_OK && host_io) {
         st = grow(&h->stage_x, &h->stage_x_bytes, (size_t)N * h->K * es);
         if (st == BSR_OK) st = grow(&h->stage_y, &h->stage_y_bytes, (size_t)N * h->M * es);
@@ -334,7 +334,7 @@ bsr_status_t bsr_spmm(bsr_handle_t h, const void *X, const float *bias, void *Y,
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const Schedule &sc = *h->sched;
 
-    bool need_grow = (size_t)sc.n_slots * (size_t)N * sc.R * 4 > h->ws_bytes ||
+    bool need_grow = (size_t)sc.n_slots * (size_t)N * sc.ex_R * 4 > h->ws_bytes ||
                      (host_io && (xbytes > h->stage_x_bytes || ybytes > h->stage_y_bytes));
     if (need_grow) {
         if (cudaStreamSynchronize(s) != cudaSuccess) { cudaGetLastError(); return BSR_ERR_CUDA; }
@@ -407,7 +407,7 @@ bsr_status_t bsr_spmm_batch(const bsr_handle_t *handles, int n, const void *X, c
     bool synced = false;
     for (int i = 0; i < n; i++) {
         Handle *h = handles[i];
-        if ((size_t)h->sched->n_slots * (size_t)N * h->sched->R * 4 <= h->ws_bytes) continue;
+        if ((size_t)h->sched->n_slots * (size_t)N * h->sched->ex_R * 4 <= h->ws_bytes) continue;
         if (!synced) {
             if (cudaStreamSynchronize(s) != cudaSuccess) { cudaGetLastError(); return BSR_ERR_CUDA; }
             synced = true;
@@ -452,13 +452,13 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
     int64_t split_rows = 0;   // rows split into pieces (the other reduce entries are empty rows)
     for (const Split &sp : sc.splits) split_rows += sp.nslot > 0;
     snprintf(buf, len,
-             "variant=%s\ndtype=%s\nR=%d\nC=%d\nexec_C=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
+             "variant=%s\ndtype=%s\nR=%d\nC=%d\nexec_R=%d\nexec_C=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
              "\nKB=%" PRId64 "\nnnzb=%" PRId64 "\ntokens_per_cta=%d\nthreads=%d\nsmem_bytes=%zu\n"
              "item_groups=%d\nitems=%zu\nsplit_len=%d\nsplit_rows=%" PRId64 "\nslots=%d\n"
              "empty_rows=%" PRId64 "\nmax_row_blocks=%" PRId64 "\nlaunches_per_call=%d\n"
              "structure_hash=%016" PRIx64 "\ncache_hit=%d\nschedule_reuses=%" PRId64
              "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\n",
-             variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_C, sc.M, sc.K,
+             variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_R, sc.ex_C, sc.M, sc.K,
              sc.MB, sc.KB, sc.nnzb, sc.tn, sc.threads, sc.smem, sc.groups, sc.items.size(),
              sc.split_len, split_rows, sc.n_slots, sc.empty_rows, sc.max_row, launches_per_call(sc),
              sc.hash, (int)h->cache_hit, (int64_t)sc.reuse_count, (int64_t)g_cache_hits,

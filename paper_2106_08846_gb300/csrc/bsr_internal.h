@@ -80,11 +80,13 @@ struct Schedule {
     int32_t *d_indptr = nullptr;        // owned copies of the structure
     int32_t *d_indices = nullptr;
 
-    // Execution structure of the tensor-core kernel when it runs narrow bf16
-    // blocks re-blocked into R x 64 tiles (ex_C = 64; zeros for absent
-    // blocks): the items and task lists refer to these tiles; vmap gives
-    // every stored block its tile and column (tile * 64 + column).
+    // Execution structure of the tensor-core kernel when it runs small bf16
+    // blocks re-blocked into max(R, 16) x 64 tiles (ex_C = 64, ex_R; zeros for
+    // absent blocks): the items and task lists refer to these tiles; vmap
+    // gives every stored block the element offset of its first value in the
+    // tile array.
     int ex_C = 1;
+    int ex_R = 1;             // execution block height (16 for blocks of fewer rows re-blocked into tiles)
     int64_t ex_nnzb = 0;
     int64_t tc_w_total = 0;   // bytes of the tensor-core kernel's packed values (all task sizes)
     std::vector<int32_t> vmap;

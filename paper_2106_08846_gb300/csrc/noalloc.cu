@@ -61,7 +61,7 @@ extern "C" bsr_status_t bsr_spmm_noalloc(bsr_handle_t h, const void *X, const fl
     if (!X || !Y) return BSR_ERR_INVALID_ARG;
     const bsr::Schedule &sc = *h->sched;
     // the split-row partials of this call must fit the scratch array
-    if ((double)sc.n_slots * (double)N * sc.R * 4.0 > (double)BSR_NOALLOC_SCRATCH_BYTES) return BSR_ERR_CAPACITY;
+    if ((double)sc.n_slots * (double)N * sc.ex_R * 4.0 > (double)BSR_NOALLOC_SCRATCH_BYTES) return BSR_ERR_CAPACITY;
     const size_t es = bsr::dtype_size(h->dt);
     const size_t xbytes = (size_t)N * h->K * es, ybytes = (size_t)N * h->M * es;
     if ((uintptr_t)X % 16 || (uintptr_t)Y % 16 || (uintptr_t)bias % 4) return BSR_ERR_ALIGNMENT;

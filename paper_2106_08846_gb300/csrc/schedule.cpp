@@ -323,28 +323,49 @@ void plan_tc(Schedule &sc) {
 // paths measured about even on 1024x1024 weights at 16384 tokens). Fills the tile
 // structure (ptr, ind) and vmap; false if the shape or density does not fit.
 bool reblock_for_tc(const Schedule &sc, std::vector<int32_t> &ptr, std::vector<int32_t> &ind,
-                    std::vector<int32_t> &vmap) {
-    if (sc.dt != BSR_BF16 || !(sc.C == 1 || sc.C == 2 || sc.C == 4 || sc.C == 8) ||
-        !(sc.R == 16 || sc.R == 32 || sc.R == 64 || sc.R == 128) || sc.K % 8 != 0 || sc.nnzb == 0)
-        return false;
-    const int64_t tw = 64 / sc.C;   // block columns per tile
-    ptr.assign((size_t)sc.MB + 1, 0);
+                    std::vector<int32_t> &vmap, int *RT_out) {
+    const bool r_ok = sc.R == 1 || sc.R == 2 || sc.R == 4 || sc.R == 8 || sc.R == 16 || sc.R == 32 ||
+                      sc.R == 64 || sc.R == 128;
+    const bool c_ok = sc.C == 1 || sc.C == 2 || sc.C == 4 || sc.C == 8 || sc.C == 16 || sc.C == 32;
+    const int RT = std::max(sc.R, 16);   // tile height: blocks of fewer rows stack 16 / R block rows
+    if (sc.dt != BSR_BF16 || !r_ok || !c_ok || sc.M % RT != 0 || sc.K % 8 != 0 || sc.nnzb == 0) return false;
+    const int64_t tw = 64 / sc.C;        // block columns per tile
+    const int64_t g = RT / sc.R;         // block rows per tile row
+    const int64_t MBT = sc.M / RT;
+    ptr.assign((size_t)MBT + 1, 0);
     ind.clear();
     vmap.assign((size_t)sc.nnzb, 0);
-    for (int64_t i = 0; i < sc.MB; i++) {
-        int64_t last = -1;
-        for (int32_t p = sc.indptr[i]; p < sc.indptr[i + 1]; p++) {
-            const int64_t t = sc.indices[p] / tw;
-            if (t != last) {
-                ind.push_back((int32_t)t);
-                last = t;
+    std::vector<int32_t> cols;
+    for (int64_t it = 0; it < MBT; it++) {
+        // the tile row's tiles: every tile column any of its block rows touches
+        cols.clear();
+        for (int64_t i = it * g; i < (it + 1) * g; i++)
+            for (int32_t p = sc.indptr[i]; p < sc.indptr[i + 1]; p++) cols.push_back((int32_t)(sc.indices[p] / tw));
+        std::sort(cols.begin(), cols.end());
+        cols.erase(std::unique(cols.begin(), cols.end()), cols.end());
+        const int64_t first = (int64_t)ind.size();
+        ind.insert(ind.end(), cols.begin(), cols.end());
+        if ((int64_t)ind.size() * RT * 64 > INT32_MAX) return false;
+        for (int64_t i = it * g; i < (it + 1) * g; i++) {
+            const int64_t row_off = (i - it * g) * sc.R;
+            for (int32_t p = sc.indptr[i]; p < sc.indptr[i + 1]; p++) {
+                const int64_t t = sc.indices[p] / tw;
+                const int64_t k = first + (std::lower_bound(cols.begin(), cols.end(), (int32_t)t) - cols.begin());
+                vmap[(size_t)p] = (int32_t)((k * RT + row_off) * 64 + (sc.indices[p] % tw) * sc.C);
             }
-            vmap[(size_t)p] = (int32_t)(((int64_t)ind.size() - 1) * 64 + (sc.indices[p] % tw) * sc.C);
         }
-        ptr[(size_t)i + 1] = (int32_t)ind.size();
-        if ((int64_t)ind.size() * 64 > INT32_MAX) return false;
+        ptr[(size_t)it + 1] = (int32_t)ind.size();
     }
-    return sc.nnzb * sc.C >= 8 * (int64_t)ind.size();
+    *RT_out = RT;
+    // Worth it when the kept elements fill enough of the tiles. A tile costs
+    // the tensor cores about the same whatever its fill (the MMA issue rate
+    // binds), while the SIMT kernel's cost follows the kept elements at a rate
+    // that grows with the block height (X reuse across a block's rows): measured
+    // on 768 x 768 bf16 weights at 80% sparsity and 1024 tokens, 16 x 64 tiles
+    // took 25 us against 42 us (1x1), 36 us (1x32), 23 us (4x4) and 19 us (8x1)
+    // on the SIMT kernel. So one-row blocks move at 1/8 fill, taller ones at 1/4.
+    const int64_t need = sc.R == 1 ? 8 : 4;
+    return sc.nnzb * sc.R * sc.C * need >= (int64_t)ind.size() * RT * 64;
 }
 
 const char *env_str(const char *name) {
@@ -367,25 +388,30 @@ bsr_status_t build_schedule(Schedule &sc) {
     const bool want_generic = force && std::string(force) == "generic";
     const bool want_xstage = force && std::string(force) == "xstage";
     sc.ex_C = sc.C;
+    sc.ex_R = sc.R;
     sc.ex_nnzb = sc.nnzb;
     std::vector<int32_t> tptr, tind;
+    int RT = sc.R;
     const bool reblock = !want_generic && !want_xstage && !tc_supports(sc.R, sc.C, sc.dt, sc.K) &&
-                         reblock_for_tc(sc, tptr, tind, sc.vmap);
+                         reblock_for_tc(sc, tptr, tind, sc.vmap, &RT);
     if (!reblock) sc.vmap.clear();
     if (!want_generic && !want_xstage && (reblock || tc_supports(sc.R, sc.C, sc.dt, sc.K))) {
         // plan on the tile structure (the user's arrays stay the cache key)
         std::vector<int32_t> uptr, uind;
-        const int uC = sc.C;
-        const int64_t unnzb = sc.nnzb, uKB = sc.KB;
+        const int uC = sc.C, uR = sc.R;
+        const int64_t unnzb = sc.nnzb, uKB = sc.KB, uMB = sc.MB;
         if (reblock) {
             uptr.swap(sc.indptr);
             uind.swap(sc.indices);
             sc.indptr.swap(tptr);
             sc.indices.swap(tind);
             sc.C = 64;
+            sc.R = RT;
+            sc.MB = sc.M / RT;
             sc.nnzb = sc.indptr.back();
             sc.KB = (sc.K + 63) / 64;
             sc.ex_C = 64;
+            sc.ex_R = RT;
             sc.ex_nnzb = sc.nnzb;
             row_stats(sc);
         }
@@ -399,8 +425,11 @@ bsr_status_t build_schedule(Schedule &sc) {
             sc.indptr.swap(uptr);
             sc.indices.swap(uind);
             sc.C = uC;
+            sc.R = uR;
+            sc.MB = uMB;
             sc.nnzb = unnzb;
             sc.KB = uKB;
+            row_stats(sc);   // the report's row statistics describe the caller's block rows
         }
     } else if (!want_generic && xstage_supports(sc.R, sc.C, sc.dt, sc.K)) {
         sc.variant = V_XSTAGE;
@@ -465,7 +494,7 @@ bsr_status_t pack_data(Handle &h) {
         if (sc.ex_C != sc.C) {
             // re-blocked: zero-filled R x 64 tiles first, then the MMA layout
             void *tiles = nullptr;
-            const size_t tbytes = (size_t)sc.ex_nnzb * sc.R * 64 * 2;
+            const size_t tbytes = (size_t)sc.ex_nnzb * sc.ex_R * 64 * 2;
             if (cudaMalloc(&tiles, tbytes) != cudaSuccess) {
                 cudaGetLastError();
                 return BSR_ERR_ALLOC;
@@ -475,7 +504,7 @@ bsr_status_t pack_data(Handle &h) {
                 e = reblock_tc_data((const uint16_t *)h.data, sc.d_vmap, sc.nnzb, sc.R, sc.C, (uint16_t *)tiles, 0);
             for (int gi = 0; gi < kTcTaskSizes && e == cudaSuccess; gi++)
                 if (sc.tc.w_off[gi] >= 0)
-                    e = pack_tc_data(tiles, sc.dt, sc.tc.d_worder[gi], (int64_t)sc.tc.worder[gi].size(), sc.R, 64,
+                    e = pack_tc_data(tiles, sc.dt, sc.tc.d_worder[gi], (int64_t)sc.tc.worder[gi].size(), sc.ex_R, 64,
                                      (unsigned char *)h.data_packed + sc.tc.w_off[gi], 0);
             if (e == cudaSuccess) e = cudaDeviceSynchronize();
             cudaFree(tiles);
@@ -555,7 +584,7 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
         if (!fits(G)) continue;
         const int64_t ctas = tiles * ((items + G - 1) / G);
         const int64_t slots = (int64_t)sc.sm_count *
-                              tc_ctas_per_sm(sc.R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt);
+                              tc_ctas_per_sm(sc.ex_R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt);
         const double waves = (double)((ctas + slots - 1) / slots);
         const double cost = waves * (kOverheadItems + (double)std::min<int64_t>(G, items));
         if (best_cost < 0 || cost < best_cost) {

@@ -90,13 +90,14 @@ cudaError_t launch_reduce(const LaunchArgs &a) {
     const Schedule &sc = *a.sc;
     const int n_splits = (int)sc.splits.size();
     if (n_splits == 0) return cudaSuccess;
-    const int64_t total = (int64_t)n_splits * a.N * sc.R;
+    const int R = sc.ex_R;   // rows per split row (tile rows of re-blocked weights)
+    const int64_t total = (int64_t)n_splits * a.N * R;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, 1 << 20));
     if (sc.dt == BSR_F32)
         return launch_kernel(k_reduce<float>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
-                             n_splits, (const float *)a.ws, a.bias, (float *)a.Y, a.N, sc.M, sc.R);
+                             n_splits, (const float *)a.ws, a.bias, (float *)a.Y, a.N, sc.M, R);
     return launch_kernel(k_reduce<uint16_t>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
-                         n_splits, (const float *)a.ws, a.bias, (uint16_t *)a.Y, a.N, sc.M, sc.R);
+                         n_splits, (const float *)a.ws, a.bias, (uint16_t *)a.Y, a.N, sc.M, R);
 }
 
 }  // namespace bsr

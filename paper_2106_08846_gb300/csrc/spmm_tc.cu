@@ -511,8 +511,7 @@ __global__ void k_reblock(const uint16_t *__restrict__ data, const int32_t *__re
         const int64_t p = e / ((int64_t)R * C);
         const int rc = (int)(e - p * R * C);
         const int r = rc / C, c = rc - r * C;
-        const int64_t v = vmap[p];
-        tiles[((v >> 6) * R + r) * 64 + (v & 63) + c] = data[e];
+        tiles[(int64_t)vmap[p] + r * 64 + c] = data[e];   // vmap: offset of the block's (0, 0) in the tiles
     }
 }
 
@@ -706,7 +705,7 @@ cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t n
 
 template <typename T>
 cudaError_t launch_tc_t(const LaunchArgs *las, const int *Gs, int n) {
-    switch (las[0].sc->R) {
+    switch (las[0].sc->ex_R) {
         case 16: return launch_r<T, 16>(las, Gs, n);
         case 32: return launch_r<T, 32>(las, Gs, n);
         case 64: return launch_r<T, 64>(las, Gs, n);
@@ -719,7 +718,7 @@ cudaError_t launch_tc(const LaunchArgs &la, int G) {
     return la.sc->dt == BSR_F32 ? launch_tc_t<float>(&la, &G, 1) : launch_tc_t<uint16_t>(&la, &G, 1);
 }
 
-int tc_fusion_key(const Schedule &sc) { return (int)sc.dt * 1024 + sc.R; }
+int tc_fusion_key(const Schedule &sc) { return (int)sc.dt * 1024 + sc.ex_R; }
 
 cudaError_t launch_tc_batch(const LaunchArgs *las, const int *Gs, int n) {
     if (n <= 0) return cudaSuccess;

@@ -94,19 +94,21 @@ def test_fp32_chain_through_every_kernel_kind():
 
 
 def test_bf16_chain_tensor_core_and_simt():
-    """bf16: 16x16 (tensor cores) -> 1x1 (xstage) -> 32x32 (tensor cores) ->
-    32x1 (re-blocked onto the tensor cores or xstage), each call's X the
-    previous call's Y."""
+    """bf16: 16x16 (tensor cores) -> sparse 1x1 (xstage) -> 32x32 (tensor
+    cores) -> dense 1x1 (re-blocked into 16-row tiles for the tensor cores) ->
+    32x1, each call's X the previous call's Y."""
     N = 333
     layers = [
         _layer(1301, 512, 256, 16, 16, "bf16", 0.3),
-        _layer(1302, 256, 512, 1, 1, "bf16", 0.2),
+        _layer(1302, 256, 512, 1, 1, "bf16", 0.06),
         _layer(1303, 512, 256, 32, 32, "bf16", 0.3),
-        _layer(1304, 256, 512, 32, 1, "bf16", 0.2),
+        _layer(1306, 256, 512, 1, 1, "bf16", 0.3),
+        _layer(1304, 512, 256, 32, 1, "bf16", 0.2),
     ]
     handles, ins, outs = _run_chain(layers, N, "bf16", 1305)
     kinds = [h.schedule()["variant"] for h in handles]
-    assert kinds[0] == "tcgen05" and kinds[1] == "xstage" and kinds[2] == "tcgen05"
+    assert kinds[:4] == ["tcgen05", "xstage", "tcgen05", "tcgen05"]
+    assert handles[3].schedule()["exec_R"] == 16
     _check(layers, ins, outs)
 
 

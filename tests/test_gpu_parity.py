@@ -346,6 +346,35 @@ def test_narrow_bf16_blocks_run_as_tensor_core_tiles(R, C):
     check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M)
 
 
+@pytest.mark.parametrize("R,C", [(1, 1), (1, 32), (4, 4), (8, 1), (2, 16), (8, 8)])
+def test_small_bf16_blocks_run_as_16_row_tensor_core_tiles(R, C):
+    """bf16 blocks of fewer than 16 rows, dense enough, stack 16 / R block rows
+    into zero-filled 16 x 64 tiles for the tensor cores; the product matches
+    the oracle on the original blocks (ragged tokens, a partial last tile,
+    rows without blocks)."""
+    M, K = 256, 64 * 5 + 32
+    MB, KB = M // R, K // C
+    cnt = np.full(MB, max(1, int(KB * 0.35)), dtype=np.int64)
+    cnt[[3, MB // 2]] = 0   # rows without blocks (their tile rows still hold other rows' blocks)
+    w = synth.make_weight("t", 70 + R + C, M, K, R, C, "bf16", 0,
+                          mask=synth.mask_from_row_counts(70 + R + C, cnt, KB))
+    X = synth.activations(71, 210, K, "bf16")
+    h, _, Y = _run(w, X)
+    s = h.schedule()
+    assert s["variant"] == "tcgen05" and s["exec_R"] == 16 and s["exec_C"] == 64
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M)
+
+
+def test_small_bf16_blocks_whose_rows_do_not_fill_tiles_stay_simt():
+    """M not a multiple of 16 (4-row blocks, M = 260): no 16-row tiling, the
+    SIMT kernel keeps the weight."""
+    w = _weight(260, 256, 4, 4, "bf16", 0.4, 80)
+    X = synth.activations(81, 100, 256, "bf16")
+    h, _, Y = _run(w, X)
+    assert h.schedule()["variant"] == "xstage"
+    check_product(Y, oracle.bsr_from_dense(w.W, 4, 4), X, w.bias, 260)
+
+
 def test_sparse_narrow_bf16_blocks_stay_simt():
     """Below about 8 kept columns per 64-column tile the padded tensor work is
     not worth it: the SIMT kernel keeps the weight."""
