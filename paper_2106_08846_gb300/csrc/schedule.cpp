@@ -13,6 +13,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <numeric>
+#include <queue>
 #include <string>
 
 #include "schedule.h"
@@ -254,11 +255,18 @@ void plan_xstage(Schedule &sc) {
     }
 }
 
+// Tasks of the tensor-core kernel for every task size G: ceil(items / G)
+// tasks of at most G items each, balanced by work (a CTA's MMAs follow its
+// blocks): the items, longest first, each go to the least-loaded task that
+// still has room (ties: the lower task). Each task's record carries its items,
+// its chunk starts and its MMA entries; its block values are packed task by
+// task, chunk by chunk.
 void plan_tc(Schedule &sc) {
     const int kc = tc_chunk_cols(sc.dt);
     const int64_t es = (int64_t)dtype_size(sc.dt);
     const int64_t nch = (sc.K + kc - 1) / kc;
     const size_t per_block = tc_block_bytes(sc.R, sc.C, sc.dt);
+    const int64_t n_items = (int64_t)sc.items.size();
     int64_t total = 0;   // bytes of packed values over all usable G
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         const int G = kTcG[gi];
@@ -268,45 +276,77 @@ void plan_tc(Schedule &sc) {
         rec.clear();
         off.clear();
         order.clear();
+        sc.tc.task_blocks_max[gi] = 0;
         size_t wmax = 0, imax = 0;
+        const int64_t n_tasks = (n_items + G - 1) / G;
+        std::vector<std::vector<int32_t>> members((size_t)n_tasks);
+        {
+            using Load = std::pair<int64_t, int64_t>;   // (blocks, task)
+            std::priority_queue<Load, std::vector<Load>, std::greater<Load>> open;
+            for (int64_t t = 0; t < n_tasks; t++) open.push({0, t});
+            for (int64_t k = 0; k < n_items; k++) {
+                const Load l = open.top();
+                open.pop();
+                members[(size_t)l.second].push_back((int32_t)k);
+                if ((int)members[(size_t)l.second].size() < G)
+                    open.push({l.first + sc.items[(size_t)k].p1 - sc.items[(size_t)k].p0, l.second});
+                else
+                    sc.tc.task_blocks_max[gi] = std::max(sc.tc.task_blocks_max[gi],
+                                                         l.first + sc.items[(size_t)k].p1 - sc.items[(size_t)k].p0);
+            }
+            while (!open.empty()) {
+                sc.tc.task_blocks_max[gi] = std::max(sc.tc.task_blocks_max[gi], open.top().first);
+                open.pop();
+            }
+        }
         std::vector<std::vector<int32_t>> per_chunk((size_t)nch), src((size_t)nch);
-        for (size_t t = 0; t < sc.items.size(); t += G) {
+        for (int64_t t = 0; t < n_tasks; t++) {
             for (auto &v : per_chunk) v.clear();
             for (auto &v : src) v.clear();
-            const size_t t_end = std::min(sc.items.size(), t + G);
-            for (size_t k = t; k < t_end; k++) {
-                const Item &it = sc.items[k];
+            const std::vector<int32_t> &mem = members[(size_t)t];
+            const int g_count = (int)mem.size();
+            for (int g = 0; g < g_count; g++) {
+                const Item &it = sc.items[(size_t)mem[(size_t)g]];
                 for (int32_t b = 0; b < it.p1 - it.p0; b++) {
                     const int64_t col = sc.indices[it.p0 + b];
                     const int64_t c = (col * sc.C) / kc;
                     const int32_t a32 = (int32_t)(((col * sc.C) % kc) * es / 32);
-                    per_chunk[(size_t)c].push_back(a32 | (int32_t)((k - t) << 2) | ((b == 0) << 7));
+                    per_chunk[(size_t)c].push_back(a32 | (g << 2) | ((b == 0) << 7));
                     src[(size_t)c].push_back(it.p0 + b);
                 }
             }
             off.push_back((int32_t)rec.size());
             const size_t head = rec.size();
-            rec.resize(head + (size_t)tc_pad4(nch + 2), 0);
-            rec[head] = (int32_t)order.size();   // the task's first packed block
+            const size_t items_at = head + 4 + (size_t)tc_pad4(nch + 1);
+            rec.resize(items_at + 4 * (size_t)g_count, 0);
+            rec[head + 0] = (int32_t)order.size();   // the task's first packed block
+            rec[head + 1] = g_count;
             int32_t n = 0;
             for (int64_t c = 0; c < nch; c++) {
-                rec[head + 1 + (size_t)c] = n;
+                rec[head + 4 + (size_t)c] = n;
                 n += (int32_t)per_chunk[(size_t)c].size();
                 wmax = std::max(wmax, per_chunk[(size_t)c].size() * per_block);
             }
-            rec[head + 1 + (size_t)nch] = n;
+            rec[head + 4 + (size_t)nch] = n;
+            for (int g = 0; g < g_count; g++) {
+                const Item &it = sc.items[(size_t)mem[(size_t)g]];
+                rec[items_at + 4 * (size_t)g + 0] = it.row;
+                rec[items_at + 4 * (size_t)g + 1] = it.p0;
+                rec[items_at + 4 * (size_t)g + 2] = it.p1;
+                rec[items_at + 4 * (size_t)g + 3] = it.slot;
+            }
             for (int64_t c = 0; c < nch; c++) {
                 rec.insert(rec.end(), per_chunk[(size_t)c].begin(), per_chunk[(size_t)c].end());
                 order.insert(order.end(), src[(size_t)c].begin(), src[(size_t)c].end());
             }
-            rec.resize(head + (size_t)tc_pad4(nch + 2) + (size_t)tc_pad4(n), 0);
+            rec.resize(items_at + 4 * (size_t)g_count + (size_t)tc_pad4(n), 0);
             imax = std::max(imax, (rec.size() - head) * 4);
         }
         sc.tc.task_wbytes[gi] = (wmax + 15) & ~size_t(15);
         sc.tc.task_ibytes[gi] = imax;
         const bool ok = G * sc.R <= kTcTmemCols &&
                         tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], imax, sc.dt) <= (size_t)kTcMaxSmem &&
-                        (int64_t)order.size() < INT32_MAX;
+                        (int64_t)order.size() < INT32_MAX && (int64_t)rec.size() < INT32_MAX;
         sc.tc.w_off[gi] = ok ? (total + 255) & ~int64_t(255) : -1;
         if (ok) total = sc.tc.w_off[gi] + (int64_t)order.size() * (int64_t)per_block;
         else order.clear();
@@ -314,14 +354,12 @@ void plan_tc(Schedule &sc) {
     sc.tc_w_total = total;
 }
 
-// Narrow bf16 blocks (R in 16..128, C in 1..8) on the tensor cores: the
-// kept blocks of each block row, grouped by 64-column tile, become dense
-// R x 64 tiles with zeros for absent blocks -- a gathered-K product whose
-// gather is replaced by zero padding. Worth it while the tiles are dense
-// enough: on average at least 8 kept columns per tile (the tensor cores do
-// 64 columns of work per tile at many times the SIMT rate; at 6.4 the two
-// paths measured about even on 1024x1024 weights at 16384 tokens). Fills the tile
-// structure (ptr, ind) and vmap; false if the shape or density does not fit.
+// Small or narrow bf16 blocks on the tensor cores: the kept blocks of each
+// group of max(R, 16) rows, grouped by 64-column tile, become dense
+// max(R, 16) x 64 tiles with zeros for absent blocks -- a gathered-K product
+// whose gather is replaced by zero padding. Worth it while the tiles are
+// dense enough (below). Fills the tile structure (ptr, ind) and vmap; false
+// if the shape or density does not fit.
 bool reblock_for_tc(const Schedule &sc, std::vector<int32_t> &ptr, std::vector<int32_t> &ind,
                     std::vector<int32_t> &vmap, int *RT_out) {
     const bool r_ok = sc.R == 1 || sc.R == 2 || sc.R == 4 || sc.R == 8 || sc.R == 16 || sc.R == 32 ||
@@ -359,12 +397,13 @@ bool reblock_for_tc(const Schedule &sc, std::vector<int32_t> &ptr, std::vector<i
     *RT_out = RT;
     // Worth it when the kept elements fill enough of the tiles. A tile costs
     // the tensor cores about the same whatever its fill (the MMA issue rate
-    // binds), while the SIMT kernel's cost follows the kept elements at a rate
-    // that grows with the block height (X reuse across a block's rows): measured
-    // on 768 x 768 bf16 weights at 80% sparsity and 1024 tokens, 16 x 64 tiles
-    // took 25 us against 42 us (1x1), 36 us (1x32), 23 us (4x4) and 19 us (8x1)
-    // on the SIMT kernel. So one-row blocks move at 1/8 fill, taller ones at 1/4.
-    const int64_t need = sc.R == 1 ? 8 : 4;
+    // binds), while the SIMT kernel's cost follows the kept elements. Measured
+    // (two tensor-core CTAs per SM): on 768 x 768 bf16 weights at 80% sparsity
+    // and 1024 tokens (fill about 0.2) the tiles took 17-19 us against the SIMT
+    // kernel's 19-42 us for every shape from 1x1 to 32x1; on a 1024 x 1024
+    // 32x1 weight at 90% with 16384 tokens (fill 0.10) 111 us against 166 us.
+    // So blocks move while they fill at least 1/12 of the tiles.
+    const int64_t need = 12;
     return sc.nnzb * sc.R * sc.C * need >= (int64_t)ind.size() * RT * 64;
 }
 
@@ -563,9 +602,12 @@ int choose_tasks(const Schedule &sc, int64_t N) {
     return best;
 }
 
-// Task size for the tcgen05 kernel: the same waves x (overhead + work) model,
-// among the G whose accumulators fit tensor memory and whose shared memory
-// fits; a wave is every SM holding as many CTAs as fit it at once.
+// Task size for the tcgen05 kernel: the G that minimises waves x (fixed CTA
+// cost + the most loaded task's MMAs), among the G whose accumulators fit
+// tensor memory and whose shared memory fits; a wave is every SM holding as
+// many CTAs as fit it at once. A CTA's fixed cost (tensor-memory allocation,
+// barriers, work list, first stage round trip, epilogue) is worth about
+// kOverheadMma MMAs.
 int choose_tc_tasks(const Schedule &sc, int64_t N) {
     static const int forced = [] {
         const char *v = getenv("BSR_TC_G");
@@ -574,19 +616,19 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
     auto fits = [&](int G) { return sc.tc.w_off[tc_g_index(G)] >= 0; };   // planned and packed for G
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (forced == kTcG[gi] && fits(forced)) return forced;
-    const double kOverheadItems = 4.0;
+    const double kOverheadMma = 32.0;
+    const double mma_per_block = sc.dt == BSR_F32 ? 3.0 * sc.ex_C / 8.0 : sc.ex_C / 16.0;
     const int64_t tiles = (N + kTcTokens - 1) / kTcTokens;
-    const int64_t items = (int64_t)sc.items.size();
     int best = 1;
     double best_cost = -1.0;
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         const int G = kTcG[gi];
         if (!fits(G)) continue;
-        const int64_t ctas = tiles * ((items + G - 1) / G);
+        const int64_t ctas = tiles * (int64_t)sc.tc.rec_off[gi].size();
         const int64_t slots = (int64_t)sc.sm_count *
                               tc_ctas_per_sm(sc.ex_R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt);
         const double waves = (double)((ctas + slots - 1) / slots);
-        const double cost = waves * (kOverheadItems + (double)std::min<int64_t>(G, items));
+        const double cost = waves * (kOverheadMma + (double)sc.tc.task_blocks_max[gi] * mma_per_block);
         if (best_cost < 0 || cost < best_cost) {
             best_cost = cost;
             best = G;

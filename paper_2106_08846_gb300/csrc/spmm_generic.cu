@@ -47,23 +47,31 @@ k_generic(const Item *__restrict__ items, int n_items, const int32_t *__restrict
     }
 }
 
-// Y[n, row*R + r] = sum over the row's pieces, in piece order, + bias.
+// Y[n, row*R + r] = sum over the row's pieces, in piece order, + bias. One
+// CTA per (split row, tile of `tn` tokens): the tile's tn x R outputs are
+// R-contiguous runs of Y, so consecutive threads write consecutive
+// addresses; index arithmetic is one 64-bit division per tile and 32-bit
+// inside it.
 template <typename T>
-__global__ void k_reduce(const Split *__restrict__ splits, int n_splits, const float *__restrict__ ws,
-                         const float *__restrict__ bias, T *__restrict__ Y, int64_t N, int64_t M, int R) {
+__global__ void __launch_bounds__(256)
+k_reduce(const Split *__restrict__ splits, int n_splits, const float *__restrict__ ws,
+         const float *__restrict__ bias, T *__restrict__ Y, int64_t N, int64_t M, int R, int tn, int64_t n_tiles) {
     ptx::pdl_launch_dependents();
     ptx::pdl_wait();   // the partials come from the product kernel just before
-    const int64_t total = (int64_t)n_splits * N * R;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t rest = e / R;
-        const int r = (int)(e - rest * R);
-        const int64_t s = rest / N, n = rest - s * N;
+    const int64_t work = (int64_t)n_splits * n_tiles;
+    for (int64_t b = blockIdx.x; b < work; b += gridDim.x) {
+        const int64_t s = b / n_tiles;
+        const int64_t n0 = (b - s * n_tiles) * tn;
         const Split sp = splits[s];
-        float acc = 0.f;
-        for (int k = 0; k < sp.nslot; k++) acc += ws[((int64_t)(sp.slot0 + k) * N + n) * R + r];
-        const int64_t m = (int64_t)sp.row * R + r;
-        Y[n * M + m] = from_f32<T>(acc + (bias ? bias[m] : 0.f));
+        const unsigned outs = (unsigned)(N - n0 < tn ? N - n0 : tn) * (unsigned)R;
+        const int64_t m0 = (int64_t)sp.row * R;
+        for (unsigned o = threadIdx.x; o < outs; o += blockDim.x) {
+            const unsigned t = o / (unsigned)R, r = o - t * (unsigned)R;
+            const int64_t n = n0 + t;
+            float acc = 0.f;
+            for (int k = 0; k < sp.nslot; k++) acc += ws[((int64_t)(sp.slot0 + k) * N + n) * R + r];
+            Y[n * M + m0 + r] = from_f32<T>(acc + (bias ? bias[m0 + r] : 0.f));
+        }
     }
 }
 
@@ -89,15 +97,16 @@ cudaError_t launch_generic(const LaunchArgs &a) {
 cudaError_t launch_reduce(const LaunchArgs &a) {
     const Schedule &sc = *a.sc;
     const int n_splits = (int)sc.splits.size();
-    if (n_splits == 0) return cudaSuccess;
+    if (n_splits == 0 || a.N == 0) return cudaSuccess;
     const int R = sc.ex_R;   // rows per split row (tile rows of re-blocked weights)
-    const int64_t total = (int64_t)n_splits * a.N * R;
-    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, 1 << 20));
+    const int tn = std::max(1, 1024 / R);   // about 1024 outputs per tile
+    const int64_t n_tiles = (a.N + tn - 1) / tn;
+    const int grid = (int)std::min<int64_t>((int64_t)n_splits * n_tiles, 1 << 20);
     if (sc.dt == BSR_F32)
         return launch_kernel(k_reduce<float>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
-                             n_splits, (const float *)a.ws, a.bias, (float *)a.Y, a.N, sc.M, R);
+                             n_splits, (const float *)a.ws, a.bias, (float *)a.Y, a.N, sc.M, R, tn, n_tiles);
     return launch_kernel(k_reduce<uint16_t>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
-                         n_splits, (const float *)a.ws, a.bias, (uint16_t *)a.Y, a.N, sc.M, R);
+                         n_splits, (const float *)a.ws, a.bias, (uint16_t *)a.Y, a.N, sc.M, R, tn, n_tiles);
 }
 
 }  // namespace bsr

@@ -25,8 +25,9 @@
 //                         adds the bias, converts and stores Y (or an fp32
 //                         partial for a split row).
 //
-// bf16 uses a 6-stage ring, one CTA per SM; fp32 a 2-stage ring (plus the low
-// twins) so that two CTAs share an SM and overlap their stage round trips.
+// Two CTAs share an SM, so that one CTA's set-up, stage round trips and
+// epilogue overlap the other's MMAs: bf16 uses a 3-stage ring, fp32 a 2-stage
+// ring (plus the low twins).
 // Launched with programmatic stream serialisation: set-up and the work list
 // come before the wait for the previous kernel; X, bias, Y after it. Every
 // wait is bounded by the global timer; a timeout sets the device status word,
@@ -63,9 +64,8 @@ constexpr int NTHREADS = NWARPS * 32;
 constexpr uint64_t kDrainNs = 200000000ull;
 
 struct TcArgs {
-    const Item *items;
-    int n_items, G, n_tasks;
-    const int32_t *trec;      // task records: chunk starts, then MMA entries
+    int G, n_tasks;           // G: most items in a task (accumulator columns G * R)
+    const int32_t *trec;      // task records: header, chunk starts, items, MMA entries
     const int32_t *trec_off;  // per task: record offset (ints)
     const void *wpk;          // block values in the MMA's B layout (fp32: high then low parts), task-chunk order
     uint32_t wstage;          // bytes of one W ring stage
@@ -174,9 +174,10 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
     const int64_t n_tiles = (a.N + TN - 1) / TN;
     const int task = (int)(cta / n_tiles);
     const int64_t n0 = (int64_t)(cta % n_tiles) * TN;
-    const int item_first = task * a.G;
-    const int g_count = min(a.G, a.n_items - item_first);
+    const int32_t *trec = a.trec + __ldg(a.trec_off + task);
+    const int g_count = __ldg(trec + 1);
     const int C = a.C, nch = a.nchunks;
+    const int items_at = 4 + pad4(nch + 1);   // record layout: header, chunk starts, items, entries
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; s++) {
@@ -191,13 +192,13 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
     }
     if ((int)threadIdx.x < g_count) {
         const int g = threadIdx.x;
-        const Item it = a.items[item_first + g];
-        itab[6 * g + 0] = it.row;
-        itab[6 * g + 1] = it.p0;
-        itab[6 * g + 2] = it.p1;
-        itab[6 * g + 3] = it.slot;
+        const int4 it = __ldg(reinterpret_cast<const int4 *>(trec + items_at) + g);   // row, p0, p1, slot
+        itab[6 * g + 0] = it.x;
+        itab[6 * g + 1] = it.y;
+        itab[6 * g + 2] = it.z;
+        itab[6 * g + 3] = it.w;
         itab[6 * g + 4] = 0;
-        itab[6 * g + 5] = it.p1 - it.p0;
+        itab[6 * g + 5] = it.z - it.y;
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -216,9 +217,8 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
         // ---------------- producer
         if (lane == 0) {
             ptx::prefetch_tensormap(&xmap);
-            const int32_t *trec = a.trec + __ldg(a.trec_off + task);
-            const int n_ent = __ldg(trec + 1 + nch);
-            const uint32_t rec_bytes = (uint32_t)(pad4(nch + 2) + pad4(n_ent)) * 4;
+            const int n_ent = __ldg(trec + 4 + nch);
+            const uint32_t rec_bytes = (uint32_t)(items_at + 4 * g_count + pad4(n_ent)) * 4;
             ptx::mbar_arrive_expect_tx(rbar, rec_bytes);
             ptx::bulk_load(I_s, trec, rec_bytes, rbar);
             ptx::pdl_wait();   // X may be an earlier kernel's output
@@ -228,7 +228,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
             bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);   // chunk starts, from shared memory
             const int64_t wfirst = ok ? I_s[0] : 0;                   // the task's first packed block
             for (int c = 0; ok && c < nch; c++) {
-                const int lo = I_s[1 + c], hi = I_s[2 + c];
+                const int lo = I_s[4 + c], hi = I_s[5 + c];
                 if (lo == hi) continue;   // no block of this task in chunk c
                 const int s = k % NS;
                 if (k >= NS && !ptx::mbar_wait_bounded(&empty[s], ((k / NS) - 1) & 1, a.wait_ns)) {
@@ -259,10 +259,10 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
         // ---------------- MMA issuer
         if (lane == 0) {
             bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns) && !aborted(misc);
-            const int32_t *ent = I_s + pad4(nch + 2);
+            const int32_t *ent = I_s + items_at + 4 * g_count;
             int k = 0;   // chunks consumed
             for (int c = 0; ok && c < nch; c++) {
-                const int lo = I_s[1 + c], hi = I_s[2 + c];
+                const int lo = I_s[4 + c], hi = I_s[5 + c];
                 if (lo == hi) continue;
                 const int s = k % NS;
                 // fp32: wait for the split parts (the split warps waited for the copy)
@@ -356,7 +356,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
             split_ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);
             int k = 0;
             for (int c = 0; split_ok && c < nch; c++) {
-                if (I_s[1 + c] == I_s[2 + c]) continue;
+                if (I_s[4 + c] == I_s[5 + c]) continue;
                 const int s = k % NS;
                 const bool got = ptx::mbar_wait_bounded(&full[s], (k / NS) & 1, a.wait_ns) && !aborted(misc);
                 if (ptx::named_barrier_or(2, 128, !got)) { split_ok = false; break; }
@@ -444,7 +444,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
 }
 
 template <typename T, int R>
-__global__ void __launch_bounds__(NTHREADS, sizeof(T) == 4 ? 2 : 1)
+__global__ void __launch_bounds__(NTHREADS, 2)
 k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
     tc_cta<T, R>(xmap, a, blockIdx.x);
 }
@@ -459,7 +459,7 @@ struct TcBatch {
 };
 
 template <typename T, int R>
-__global__ void __launch_bounds__(NTHREADS, sizeof(T) == 4 ? 2 : 1)
+__global__ void __launch_bounds__(NTHREADS, 2)
 k_tc_batch(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ TcBatch b) {
     int h = 0;
     while (h + 1 < b.n && blockIdx.x >= b.start[h + 1]) h++;
@@ -547,10 +547,8 @@ cudaError_t make_tc_args(const LaunchArgs &la, int G, TcArgs &a, uint32_t &smem)
     smem = 0;
     if (n_items == 0 || la.N == 0) return cudaSuccess;
     const int gidx = tc_g_index(G);
-    a.items = sc.d_items;
-    a.n_items = n_items;
     a.G = G;
-    a.n_tasks = (n_items + G - 1) / G;
+    a.n_tasks = (int)sc.tc.rec_off[gidx].size();
     a.trec = sc.tc.d_rec[gidx];
     a.trec_off = sc.tc.d_rec_off[gidx];
     if (sc.tc.w_off[gidx] < 0) return cudaErrorInvalidConfiguration;
@@ -678,7 +676,7 @@ int tc_ctas_per_sm(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt) {
     const size_t per_cta = tc_smem_bytes(R, G, wbytes, ibytes, dt) + 1024;
     const int by_smem = (int)(kSmemPerSm / per_cta);
     const int by_tmem = kTcTmemCols / (int)tmem_cols_for(G * R);
-    const int bound = dt == BSR_F32 ? 2 : 1;   // the kernel's __launch_bounds__
+    const int bound = 2;   // the kernel's __launch_bounds__
     return std::max(1, std::min(bound, std::min(by_smem, by_tmem)));
 }
 

@@ -11,7 +11,7 @@ namespace bsr {
 
 constexpr int kTcTokens = 128;         // tokens per CTA = MMA M = TMEM lanes
 constexpr int kTcChunk = 64;           // K columns per ring stage (one 128-byte swizzle row of bf16)
-constexpr int kTcStages = 6;           // ring depth (bf16)
+constexpr int kTcStages = 3;           // ring depth (bf16; two CTAs per SM)
 constexpr int kTcStagesF32 = 2;        // ring depth (fp32: each stage has a twin for the low parts; two
                                        // stages let two CTAs share an SM and overlap their stage latencies)
 constexpr int kTcMaxSmem = 232448;     // 227 KB
@@ -29,6 +29,7 @@ constexpr int kTcG[kTcTaskSizes] = {1, 2, 4, 8, 16, 32};
 struct TcPlan {
     size_t task_wbytes[kTcTaskSizes] = {};   // W ring stage bytes
     size_t task_ibytes[kTcTaskSizes] = {};
+    int64_t task_blocks_max[kTcTaskSizes] = {};   // blocks of the most loaded task
     std::vector<int32_t> rec[kTcTaskSizes];       // all task records of this G
     std::vector<int32_t> rec_off[kTcTaskSizes];   // per task: offset (ints, multiple of 4)
     std::vector<int32_t> worder[kTcTaskSizes];    // per packed block: the (execution) block it holds
@@ -38,11 +39,12 @@ struct TcPlan {
     int32_t *d_worder[kTcTaskSizes] = {};
 };
 
-// A task record (int32): [ the task's first packed block, then per K chunk
-// c = 0..nchunks the index of the chunk's first entry, padded to 4 | one
-// entry per MMA-block, chunk by chunk, padded to 4 ]. Entry e uses packed
-// block (first + e). Entry bits: [0,2) stage column offset / 32 bytes,
-// [2,7) item in the task, 7 first block of its item.
+// A task record (int32): [ the task's first packed block, its item count g,
+// 0, 0 | per K chunk c = 0..nchunks the index of the chunk's first entry,
+// padded to 4 | per item (row, p0, p1, slot) | one entry per MMA-block,
+// chunk by chunk, padded to 4 ]. Entry e uses packed block (first + e).
+// Entry bits: [0,2) stage column offset / 32 bytes, [2,7) item in the task,
+// 7 first block of its item.
 inline int64_t tc_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
 bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K);

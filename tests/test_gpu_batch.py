@@ -60,7 +60,7 @@ def _run_both(ws, N, dtype, seed, with_bias=True):
     return hs, X, [to_host(y) for y in Yb], [to_host(y) for y in Ys]
 
 
-DENSE, SPARSE = (0.5, 0.3, 0.2), (0.1, 0.06, 0.03)
+DENSE, SPARSE = (0.5, 0.3, 0.2), (0.06, 0.04, 0.02)   # SPARSE: bf16 narrow blocks stay SIMT below 1/12 fill
 
 
 @pytest.mark.parametrize("R,C,dtype,dens,kind", [(32, 1, "f32", DENSE, "xstage"), (1, 1, "f32", DENSE, "xstage"),

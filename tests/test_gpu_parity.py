@@ -376,8 +376,8 @@ def test_small_bf16_blocks_whose_rows_do_not_fill_tiles_stay_simt():
 
 
 def test_sparse_narrow_bf16_blocks_stay_simt():
-    """Below about 8 kept columns per 64-column tile the padded tensor work is
-    not worth it: the SIMT kernel keeps the weight."""
+    """Below about 5 kept columns per 64-column tile (1/12 fill) the padded
+    tensor work is not worth it: the SIMT kernel keeps the weight."""
     w = _weight(256, 1024, 32, 1, "bf16", 0.02, 60)
     X = synth.activations(61, 64, 1024, "bf16")
     h, _, Y = _run(w, X)
