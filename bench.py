@@ -20,7 +20,16 @@ with pinned host X and Y (the library copies in and out on the call's stream;
 each weight's calls on a stream of their own).
 ``cpu_baseline`` times the CPU oracle on the host cores.
 
+``--workload 1|3|4|5`` instead reports another benchmark workload (one JSON
+line per block shape and dtype): its step as the workload defines it (one
+bsr_spmm call per weight, in order, on one stream; L2 flushed before every
+step), GFLOP/s and GB/s, and the fraction of the workload's roofline, the
+slower of its FLOPs at the arithmetic peak (fp32: the FP32 FMA peak; bf16:
+the measured bf16 tensor peak) and its bytes (block values, indices, indptr,
+X, Y, bias, each once per call) at the measured HBM bandwidth.
+
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+    python bench.py --workload 4 [--steps K]
 """
 from __future__ import annotations
 
@@ -55,6 +64,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer pass (profiling runs)")
     ap.add_argument("--shapes", default="", help="comma-separated subset of block shapes, e.g. 1x1,32x1 (profiling runs)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--workload", type=int, default=2, choices=[1, 2, 3, 4, 5],
+                    help="2: the block-shape sweep (the benchmark line); 1, 3, 4, 5: a per-workload report "
+                         "(one JSON line per block shape and dtype, device time against the roofline), 1 GPU")
     return ap.parse_args()
 
 
@@ -436,8 +448,108 @@ def run_ours(args, world, rank, local):
         h.destroy()
 
 
+REPORT_VARIANTS = {
+    1: [(None, None)],
+    3: [(None, None)],
+    4: [("f32", (32, 1)), ("f32", (16, 16)), ("bf16", (32, 1)), ("bf16", (16, 16))],
+    5: [(None, (32, 1)), (None, (16, 16))],
+}
+
+
+def run_report(args):
+    """One JSON line per block shape and dtype of workload 1, 3, 4 or 5."""
+    import torch
+
+    import synth
+    import paper_2106_08846_gb300 as bsr
+    from paper_2106_08846_gb300 import _build
+
+    _build.build()
+    bsr.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    pk = peaks()
+    props = torch.cuda.get_device_properties(dev)
+    mhz = float(pk.get("sm_max_mhz", 2070.0))
+    fp32_peak = props.multi_processor_count * FP32_LANES_PER_SM * 2 * mhz * 1e6   # FLOP/s
+    bf16_peak = float(pk["bf16_tflops"]) * 1e12
+    hbm = float(pk["hbm_gbs"]) * 1e9
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def dev_array(a):
+        if a.dtype == np.uint16:
+            return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+        return torch.from_numpy(a).to(dev)
+
+    for dt, shape in REPORT_VARIANTS[args.workload]:
+        wl = synth.config(args.workload, dtype=dt, shape=shape)
+        N, es = wl.N, (2 if wl.dtype == "bf16" else 4)
+        X = dev_array(wl.make_X())
+        handles, biases, flops, nbytes, roof_s = [], [], [], [], []
+        peak = bf16_peak if wl.dtype == "bf16" else fp32_peak
+        for w in wl.weights:
+            arrays = bsr.bsr_from_dense(dev_array(w.W), w.R, w.C, 0.0)
+            h = bsr.bsr_create(*arrays, w.R, w.C, w.M, w.K)
+            h.reserve(N)
+            handles.append(h)
+            biases.append(torch.from_numpy(w.bias).to(dev))
+            flops.append(2 * N * w.nnz)
+            nbytes.append(workload_bytes(w, N, es))
+            roof_s.append(max(flops[-1] / peak, nbytes[-1] / hbm))
+        Y = torch.empty((N, wl.weights[0].M), dtype=X.dtype, device=dev)   # every weight of a workload is M x K
+        scheds = [h.schedule() for h in handles]
+
+        def step():
+            for h, b in zip(handles, biases):
+                bsr.bsr_spmm(h, X, b, Y, N, stream)
+
+        for _ in range(max(args.warmup, 3)):
+            flush.zero_()
+            step()
+        torch.cuda.synchronize()
+        K = max(1, args.steps)
+        st = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+        with ClockSampler(0) as clocks:
+            for k in range(K):
+                flush.zero_()
+                st[k][0].record(stream)
+                step()
+                st[k][1].record(stream)
+            torch.cuda.synchronize()
+        for h in handles:
+            if h.check_device_status() != 0:
+                raise RuntimeError("device status error during the report")
+        step_s = statistics.median(a.elapsed_time(b) for a, b in st) * 1e-3
+        variants = sorted({sc["variant"] + (f" (exec {sc['exec_R']}x{sc['exec_C']})"
+                                             if (sc["exec_R"], sc["exec_C"]) != (sc["R"], sc["C"]) else "")
+                           for sc in scheds})
+        w0 = wl.weights[0]
+        line = {
+            "workload": args.workload, "name": wl.name, "shape": f"{w0.R}x{w0.C}", "dtype": wl.dtype, "N": N,
+            "M": w0.M, "K": w0.K, "weights": len(wl.weights), "calls_per_step": len(handles),
+            "variants": variants, "steps": K, "us_per_step": step_s * 1e6,
+            "gflops": sum(flops) / step_s / 1e9, "gbs": sum(nbytes) / step_s / 1e9,
+            "roofline": {"us_per_step": sum(roof_s) * 1e6, "frac": sum(roof_s) / step_s,
+                         "bound": "bytes" if sum(b / hbm for b in nbytes) >= sum(f / peak for f in flops) else "flops",
+                         "peak_tflops": peak / 1e12, "hbm_gbs": hbm / 1e9,
+                         "peak_source": ("bf16 tensor, " if wl.dtype == "bf16" else "FP32 FMA, derived from ") +
+                                        f"{pk['source']} peaks"},
+            "l2": "flushed before every step", "clocks": clocks.summary(), "data": "synthetic",
+        }
+        print(json.dumps(line), flush=True)
+        for h in handles:
+            h.destroy()
+
+
 def main():
     args = parse()
+    if args.workload != 2:
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable": "the per-workload report times the GPU path only"}))
+            return
+        run_report(args)
+        return
     world, rank, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, world, rank)
