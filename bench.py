@@ -517,10 +517,41 @@ def run_report(args):
                 step()
                 st[k][1].record(stream)
             torch.cuda.synchronize()
+        step_s = statistics.median(a.elapsed_time(b) for a, b in st) * 1e-3
+        # host time to enqueue one step as separate calls
+        t0 = time.perf_counter()
+        step()
+        host_calls_s = time.perf_counter() - t0
+        torch.cuda.synchronize()
+        plans = {}
+        if len(handles) > 1:
+            # the same step as one captured plan: the call sequence kept, and
+            # (the products being independent) regrouped and fused
+            for key, indep in (("plan_sequence", False), ("plan_fused", True)):
+                plan = bsr.bsr_plan_create(handles, [X] * len(handles), biases, [Y] * len(handles) if not indep else
+                                           [torch.empty_like(Y) for _ in handles], independent=indep)
+                for _ in range(3):
+                    flush.zero_()
+                    plan.launch(stream)
+                torch.cuda.synchronize()
+                pe = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+                for k in range(K):
+                    flush.zero_()
+                    pe[k][0].record(stream)
+                    plan.launch(stream)
+                    pe[k][1].record(stream)
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
+                plan.launch(stream)
+                host_s = time.perf_counter() - t0
+                torch.cuda.synchronize()
+                order, call, n_kernels = plan.order()
+                plans[key] = {"us_per_step": statistics.median(a.elapsed_time(b) for a, b in pe) * 1e3,
+                              "library_calls": len(set(call)), "kernels": n_kernels, "host_us": host_s * 1e6}
+                plan.destroy()
         for h in handles:
             if h.check_device_status() != 0:
                 raise RuntimeError("device status error during the report")
-        step_s = statistics.median(a.elapsed_time(b) for a, b in st) * 1e-3
         variants = sorted({sc["variant"] + (f" (exec {sc['exec_R']}x{sc['exec_C']})"
                                              if (sc["exec_R"], sc["exec_C"]) != (sc["R"], sc["C"]) else "")
                            for sc in scheds})
@@ -535,8 +566,10 @@ def run_report(args):
                          "peak_tflops": peak / 1e12, "hbm_gbs": hbm / 1e9,
                          "peak_source": ("bf16 tensor, " if wl.dtype == "bf16" else "FP32 FMA, derived from ") +
                                         f"{pk['source']} peaks"},
+            "host_us_per_step_calls": host_calls_s * 1e6,
             "l2": "flushed before every step", "clocks": clocks.summary(), "data": "synthetic",
         }
+        line.update(plans)
         print(json.dumps(line), flush=True)
         for h in handles:
             h.destroy()

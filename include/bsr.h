@@ -58,6 +58,7 @@ typedef enum {
 typedef enum { BSR_F32 = 0, BSR_BF16 = 1 } bsr_dtype_t;
 
 typedef struct bsr_handle_s *bsr_handle_t;
+typedef struct bsr_plan_s *bsr_plan_t;
 
 /*
  * bsr_from_dense -- build the BSR arrays of a dense weight on the GPU
@@ -205,6 +206,66 @@ bsr_status_t bsr_spmm_noalloc(bsr_handle_t h, const void *X, const float *bias, 
  */
 bsr_status_t bsr_spmm_batch(const bsr_handle_t *handles, int n, const void *X, const float *const *biases,
                             void *const *Ys, int64_t N, void *stream);
+
+/*
+ * bsr_plan_create -- a fixed sequence of n products, Y_i = X_i · W_iᵀ + b_i,
+ * captured once into a CUDA graph that bsr_plan_launch replays.
+ *
+ * Section 2.2: the task scheduler keeps BSR tasks in a buffer, reuses
+ * identical tasks and schedules similar ones next to each other. Identical
+ * structures already share one schedule (bsr_create's cache); a plan adds the
+ * adjacency for a whole sequence, such as every projection of a BERT model
+ * (Section 2.3), and removes the per-call host work: validation, workspace
+ * sizing and launch set-up happen here, once.
+ *
+ *   handles[n]   the weights (a handle may appear more than once); all on the
+ *                current device, which must be the one they were created on.
+ *                Each must outlive the plan (the plan uses its block values
+ *                and status word); the plan owns its split-row workspaces, so
+ *                later bsr_spmm calls on the same handles do not disturb it.
+ *   X[n]         device, [N_i, K_i] row-major, 16-byte aligned.
+ *   biases       NULL (no bias) or n entries, each NULL or device fp32 [M_i].
+ *   Y[n]         device, [N_i, M_i] row-major, 16-byte aligned; Y_i must not
+ *                overlap X_i or b_i.
+ *   N[n]         tokens per product (>= 0; 0 is a no-op product).
+ *   independent  0: the products run in the given order, one call each, so a
+ *                later X may be an earlier Y (a chain of layers).
+ *                1: the caller states that no product reads what another
+ *                writes -- checked: no Y_i may overlap any X_j, b_j or other
+ *                Y_j (BSR_ERR_INVALID_ARG otherwise) -- and the plan may
+ *                reorder: products that share X and N are grouped in first-
+ *                appearance order of their X, inside a group products whose
+ *                kernels share a template come next to each other (handles
+ *                that share a schedule adjacent) and run as fused grids as in
+ *                bsr_spmm_batch (a handle repeated inside a group starts a new
+ *                fused call). Outputs are bit-identical to bsr_spmm calls.
+ *   out          receives the plan.
+ *
+ * The buffers are bound at capture: a replay reads the current contents of
+ * X_i and b_i and writes Y_i. Synchronous (allocates the workspaces, captures
+ * on a private stream); enqueues no device work. Errors: BSR_ERR_INVALID_ARG
+ * (NULL, negative N, aliasing, host or foreign-device pointers),
+ * BSR_ERR_ALIGNMENT, BSR_ERR_ALLOC, BSR_ERR_CUDA (capture or instantiation).
+ */
+bsr_status_t bsr_plan_create(const bsr_handle_t *handles, const void *const *X, const float *const *biases,
+                             void *const *Y, const int64_t *N, int n, int independent, bsr_plan_t *out);
+
+/* bsr_plan_launch -- replay the plan's graph on `stream` (asynchronous; the
+ * products' device-side errors are reported per handle by
+ * bsr_check_device_status). Two replays of one plan must not overlap in time
+ * (they share the plan's workspaces). */
+bsr_status_t bsr_plan_launch(bsr_plan_t plan, void *stream);
+
+/* bsr_plan_get_order -- what the plan runs: order[k] = the product executed
+ * k-th and call[k] = the index of the library call (one bsr_spmm, or one
+ * fused bsr_spmm_batch group) that runs it, for k < n; products with N = 0
+ * run nothing and are not listed, entries past the executed products are -1
+ * (either array may be NULL); *n_kernels (if not NULL) = the kernel launches
+ * in the graph. */
+bsr_status_t bsr_plan_get_order(bsr_plan_t plan, int *order, int *call, int n, int *n_kernels);
+
+/* bsr_plan_destroy -- release the graph and the workspaces. NULL is a no-op. */
+void bsr_plan_destroy(bsr_plan_t plan);
 
 /* bsr_destroy -- release what the handle owns (not the borrowed arrays). NULL is a no-op. */
 void bsr_destroy(bsr_handle_t h);

@@ -66,6 +66,16 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.bsr_spmm_batch.argtypes = [ctypes.POINTER(P), ctypes.c_int, P, ctypes.POINTER(P), ctypes.POINTER(P),
                                        I64, P]
         lib.bsr_spmm_batch.restype = U
+        lib.bsr_plan_create.argtypes = [ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(P),
+                                        ctypes.POINTER(I64), ctypes.c_int, ctypes.c_int, ctypes.POINTER(P)]
+        lib.bsr_plan_create.restype = U
+        lib.bsr_plan_launch.argtypes = [P, P]
+        lib.bsr_plan_launch.restype = U
+        lib.bsr_plan_get_order.argtypes = [P, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_int), ctypes.c_int,
+                                           ctypes.POINTER(ctypes.c_int)]
+        lib.bsr_plan_get_order.restype = U
+        lib.bsr_plan_destroy.argtypes = [P]
+        lib.bsr_plan_destroy.restype = None
         lib.bsr_check_device_status.argtypes = [P]
         lib.bsr_check_device_status.restype = U
         lib.bsr_get_schedule.argtypes = [P, ctypes.c_char_p, ctypes.c_size_t]
@@ -250,6 +260,72 @@ def bsr_spmm_batch(handles, X: torch.Tensor, biases, Ys, N: Optional[int] = None
     yarr = (P * max(n, 1))(*[_ptr(Y) for Y in Ys])
     barr = None if biases is None else (P * max(n, 1))(*[_ptr(b) for b in biases])
     _check(load().bsr_spmm_batch(harr, n, _ptr(X), barr, yarr, N, _stream(stream)), "bsr_spmm_batch")
+
+
+class Plan:
+    """A product sequence captured into a CUDA graph (bsr_plan_create). Keeps
+    the handles and tensors it was built on alive."""
+
+    def __init__(self, ptr, n, keep):
+        self._ptr = ptr
+        self.n = n
+        self._keep = keep
+
+    def launch(self, stream=None) -> None:
+        _check(load().bsr_plan_launch(self._ptr, _stream(stream)), "bsr_plan_launch")
+
+    def order(self):
+        """(order, call, n_kernels): the product executed k-th, the library call
+        that runs it, and the kernel launches in the graph."""
+        n = max(self.n, 1)
+        o, c, k = (ctypes.c_int * n)(), (ctypes.c_int * n)(), ctypes.c_int(0)
+        _check(load().bsr_plan_get_order(self._ptr, o, c, self.n, ctypes.byref(k)), "bsr_plan_get_order")
+        run = [i for i in range(self.n) if o[i] >= 0]
+        return [o[i] for i in run], [c[i] for i in run], k.value
+
+    def destroy(self) -> None:
+        if self._ptr is not None:
+            load().bsr_plan_destroy(self._ptr)
+            self._ptr = None
+            self._keep = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def bsr_plan_create(handles, Xs, biases, Ys, Ns=None, independent: bool = False) -> Plan:
+    """Captures the products Ys[i] = Xs[i] W_i^T + biases[i] (device tensors)
+    into one CUDA graph; with ``independent`` the plan may regroup and fuse
+    them (see include/bsr.h)."""
+    n = len(handles)
+    if len(Xs) != n or len(Ys) != n or (biases is not None and len(biases) != n):
+        raise ValueError("one X, Y (and bias, if given) per handle")
+    Ns = [X.shape[0] for X in Xs] if Ns is None else list(Ns)
+    for h, X, Y, N in zip(handles, Xs, Ys, Ns):
+        if X.dtype != h.dtype or Y.dtype != h.dtype:
+            raise TypeError("X and Y must have the handle's dtype")
+        if not X.is_contiguous() or not Y.is_contiguous():
+            raise ValueError("X and Y must be contiguous")
+        if X.shape[-1] != h.K or Y.shape[-1] != h.M or X.shape[0] < N or Y.shape[0] < N:
+            raise ValueError("X must be [N, K] and Y [N, M]")
+    if biases is not None:
+        for b in biases:
+            if b is not None and (b.dtype != torch.float32 or not b.is_contiguous()):
+                raise TypeError("biases must be contiguous float32 tensors")
+    P = ctypes.c_void_p
+    m = max(n, 1)
+    harr = (P * m)(*[h.ptr for h in handles])
+    xarr = (P * m)(*[_ptr(X) for X in Xs])
+    yarr = (P * m)(*[_ptr(Y) for Y in Ys])
+    barr = None if biases is None else (P * m)(*[_ptr(b) for b in biases])
+    narr = (ctypes.c_int64 * m)(*Ns)
+    out = P()
+    _check(load().bsr_plan_create(harr, xarr, barr, yarr, narr, n, int(bool(independent)), ctypes.byref(out)),
+           "bsr_plan_create")
+    return Plan(out, n, (list(handles), list(Xs), list(Ys), None if biases is None else list(biases)))
 
 
 def bsr_check_device_status(h: Handle) -> int:

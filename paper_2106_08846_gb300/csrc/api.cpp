@@ -14,6 +14,7 @@
 #include <cstring>
 #include <new>
 #include <unordered_map>
+#include <vector>
 
 #include "bsr_internal.h"
 #include "schedule.h"
@@ -131,6 +132,83 @@ Schedule::~Schedule() {
 }  // namespace bsr
 
 using namespace bsr;
+
+// A captured product sequence (bsr_plan_create).
+struct bsr_plan_s {
+    int device = 0;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    std::vector<int> order, call;   // execution order; library call of each executed product
+    int n_kernels = 0;
+    std::vector<float *> ws;        // owned split-row workspaces
+    ~bsr_plan_s() {
+        DeviceGuard g(device);
+        if (exec) cudaGraphExecDestroy(exec);
+        if (graph) cudaGraphDestroy(graph);
+        for (float *p : ws) cudaFree(p);
+    }
+};
+
+namespace {
+
+// The execution order and call grouping of a plan: `calls` lists, per library
+// call, the products it runs.
+void plan_order(const bsr_handle_t *handles, const void *const *X, const int64_t *N, int n, bool independent,
+                std::vector<std::vector<int>> &calls) {
+    calls.clear();
+    if (!independent) {
+        for (int i = 0; i < n; i++)
+            if (N[i] > 0) calls.push_back({i});
+        return;
+    }
+    // groups of products sharing (X, N, dtype, K), in first-appearance order
+    std::vector<std::vector<int>> groups;
+    for (int i = 0; i < n; i++) {
+        if (N[i] == 0) continue;
+        const Handle *h = handles[i];
+        size_t g = 0;
+        for (; g < groups.size(); g++) {
+            const int j = groups[g][0];
+            if (X[j] == X[i] && N[j] == N[i] && handles[j]->dt == h->dt && handles[j]->K == h->K) break;
+        }
+        if (g == groups.size()) groups.emplace_back();
+        groups[g].push_back(i);
+    }
+    for (std::vector<int> &grp : groups) {
+        // kernels that share a template next to each other (generic last),
+        // handles that share a schedule adjacent, then the given order
+        std::vector<const Schedule *> first_seen;
+        auto sched_rank = [&](const Schedule *sc) {
+            for (size_t k = 0; k < first_seen.size(); k++)
+                if (first_seen[k] == sc) return (int)k;
+            first_seen.push_back(sc);
+            return (int)first_seen.size() - 1;
+        };
+        std::vector<std::pair<std::pair<int, int>, int>> keyed;
+        for (int i : grp) {
+            int G = 0;
+            const int fc = fusion_class(*handles[i]->sched, N[i], &G);
+            keyed.push_back({{fc < 0 ? INT32_MAX : fc, sched_rank(handles[i]->sched.get())}, i});
+        }
+        std::stable_sort(keyed.begin(), keyed.end(),
+                         [](const auto &a, const auto &b) { return a.first < b.first; });
+        // a handle may run once per call (its status word and schedule state)
+        std::vector<int> cur;
+        for (const auto &kv : keyed) {
+            const int i = kv.second;
+            bool repeat = false;
+            for (int j : cur) repeat |= handles[j] == handles[i];
+            if (repeat) {
+                calls.push_back(cur);
+                cur.clear();
+            }
+            cur.push_back(i);
+        }
+        if (!cur.empty()) calls.push_back(cur);
+    }
+}
+
+}  // namespace
 
 extern "C" {
 
@@ -429,6 +507,133 @@ bsr_status_t bsr_spmm_batch(const bsr_handle_t *handles, int n, const void *X, c
     }
     return BSR_OK;
 }
+
+bsr_status_t bsr_plan_create(const bsr_handle_t *handles, const void *const *X, const float *const *biases,
+                             void *const *Y, const int64_t *N, int n, int independent, bsr_plan_t *out) {
+    if (!out || n < 0) return BSR_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (n > 0 && (!handles || !X || !Y || !N)) return BSR_ERR_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return BSR_ERR_CUDA; }
+    std::vector<size_t> xb((size_t)n), yb((size_t)n);
+    for (int i = 0; i < n; i++) {
+        const Handle *h = handles[i];
+        if (!h || N[i] < 0 || h->device != dev) return BSR_ERR_INVALID_ARG;
+        if (N[i] == 0) continue;
+        const float *b = biases ? biases[i] : nullptr;
+        if (!X[i] || !Y[i]) return BSR_ERR_INVALID_ARG;
+        if ((uintptr_t)X[i] % 16 || (uintptr_t)Y[i] % 16 || (uintptr_t)b % 4) return BSR_ERR_ALIGNMENT;
+        const size_t es = dtype_size(h->dt);
+        xb[(size_t)i] = (size_t)N[i] * h->K * es;
+        yb[(size_t)i] = (size_t)N[i] * h->M * es;
+        if (overlaps(X[i], xb[(size_t)i], Y[i], yb[(size_t)i]) || (b && overlaps(b, (size_t)h->M * 4, Y[i], yb[(size_t)i])))
+            return BSR_ERR_INVALID_ARG;
+        if ((xb[(size_t)i] && classify(X[i], dev) != PK_DEVICE) || (yb[(size_t)i] && classify(Y[i], dev) != PK_DEVICE) ||
+            (b && classify(b, dev) != PK_DEVICE))
+            return BSR_ERR_INVALID_ARG;
+    }
+    if (independent) {
+        // no product may write what another reads or writes
+        for (int i = 0; i < n; i++) {
+            if (N[i] == 0) continue;
+            for (int j = 0; j < n; j++) {
+                if (j == i || N[j] == 0) continue;
+                const float *bj = biases ? biases[j] : nullptr;
+                if (overlaps(Y[i], yb[(size_t)i], X[j], xb[(size_t)j]) ||
+                    (bj && overlaps(Y[i], yb[(size_t)i], bj, (size_t)handles[j]->M * 4)) ||
+                    (j < i && overlaps(Y[i], yb[(size_t)i], Y[j], yb[(size_t)j])))
+                    return BSR_ERR_INVALID_ARG;
+            }
+        }
+    }
+    std::vector<std::vector<int>> calls;
+    plan_order(handles, X, N, n, independent != 0, calls);
+
+    bsr_plan_s *plan = new (std::nothrow) bsr_plan_s;
+    if (!plan) return BSR_ERR_ALLOC;
+    plan->device = dev;
+    std::vector<float *> ws_of((size_t)n, nullptr);
+    for (int i = 0; i < n; i++) {
+        if (N[i] == 0) continue;
+        const Schedule &sc = *handles[i]->sched;
+        const size_t bytes = (size_t)sc.n_slots * (size_t)N[i] * sc.ex_R * 4;
+        if (!bytes) continue;
+        if (cudaMalloc((void **)&ws_of[(size_t)i], bytes) != cudaSuccess) {
+            cudaGetLastError();
+            delete plan;
+            return BSR_ERR_ALLOC;
+        }
+        plan->ws.push_back(ws_of[(size_t)i]);
+    }
+    cudaStream_t cs = nullptr;
+    if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        delete plan;
+        return BSR_ERR_CUDA;
+    }
+    bool ok = cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed) == cudaSuccess;
+    std::vector<LaunchArgs> as;
+    for (size_t c = 0; ok && c < calls.size(); c++) {
+        as.clear();
+        for (int i : calls[c]) {
+            const Handle *h = handles[i];
+            as.push_back(LaunchArgs{h->sched.get(), h->data_packed ? h->data_packed : h->data, X[i],
+                                    biases ? biases[i] : nullptr, Y[i], ws_of[(size_t)i], h->d_status, N[i], cs,
+                                    h->wait_ns, h->stall_chunk});
+            plan->order.push_back(i);
+            plan->call.push_back((int)c);
+        }
+        ok = (as.size() == 1 ? launch_spmm(as[0]) : launch_spmm_batch(as.data(), (int)as.size())) == cudaSuccess;
+    }
+    cudaGraph_t graph = nullptr;
+    const bool ended = cudaStreamEndCapture(cs, &graph) == cudaSuccess;
+    ok = ok && ended && graph;
+    if (ok) {
+        size_t nn = 0;
+        ok = cudaGraphGetNodes(graph, nullptr, &nn) == cudaSuccess;
+        std::vector<cudaGraphNode_t> nodes(nn);
+        if (ok && nn) ok = cudaGraphGetNodes(graph, nodes.data(), &nn) == cudaSuccess;
+        for (size_t k = 0; ok && k < nn; k++) {
+            cudaGraphNodeType t;
+            ok = cudaGraphNodeGetType(nodes[k], &t) == cudaSuccess;
+            plan->n_kernels += ok && t == cudaGraphNodeTypeKernel;
+        }
+    }
+    plan->graph = graph;
+    if (ok) ok = cudaGraphInstantiate(&plan->exec, graph, 0) == cudaSuccess;
+    cudaStreamDestroy(cs);
+    if (!ok) {
+        cudaGetLastError();
+        delete plan;
+        return BSR_ERR_CUDA;
+    }
+    *out = plan;
+    return BSR_OK;
+}
+
+bsr_status_t bsr_plan_launch(bsr_plan_t plan, void *stream) {
+    if (!plan) return BSR_ERR_INVALID_ARG;
+    DeviceGuard g(plan->device);
+    if (!g.ok) return BSR_ERR_CUDA;
+    if (cudaGraphLaunch(plan->exec, static_cast<cudaStream_t>(stream)) != cudaSuccess) {
+        cudaGetLastError();
+        return BSR_ERR_CUDA;
+    }
+    return BSR_OK;
+}
+
+bsr_status_t bsr_plan_get_order(bsr_plan_t plan, int *order, int *call, int n, int *n_kernels) {
+    if (!plan || n < 0) return BSR_ERR_INVALID_ARG;
+    for (int k = 0; k < n; k++) {
+        const bool run = k < (int)plan->order.size();
+        if (order) order[k] = run ? plan->order[(size_t)k] : -1;
+        if (call) call[k] = run ? plan->call[(size_t)k] : -1;
+    }
+    if (n_kernels) *n_kernels = plan->n_kernels;
+    return BSR_OK;
+}
+
+void bsr_plan_destroy(bsr_plan_t plan) { delete plan; }
 
 bsr_status_t bsr_check_device_status(bsr_handle_t h) {
     if (!h) return BSR_ERR_INVALID_ARG;

@@ -637,21 +637,21 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
     return best;
 }
 
+int fusion_class(const Schedule &sc, int64_t N, int *G) {
+    if (sc.variant == V_XSTAGE) {
+        *G = choose_tasks(sc, N);
+        return 2 * xstage_fusion_key(sc, *G);
+    }
+    if (sc.variant == V_TC) {
+        *G = choose_tc_tasks(sc, N);
+        return 2 * tc_fusion_key(sc) + 1;
+    }
+    *G = 0;
+    return -1;
+}
+
 cudaError_t launch_spmm_batch(const LaunchArgs *as, int n) {
-    // a product's fusion class: its kernel family and the key within it
-    // (-1: runs alone), and its task size for this call
-    auto fusion = [](const LaunchArgs &a, int *G) {
-        if (a.sc->variant == V_XSTAGE) {
-            *G = choose_tasks(*a.sc, a.N);
-            return 2 * xstage_fusion_key(*a.sc, *G);
-        }
-        if (a.sc->variant == V_TC) {
-            *G = choose_tc_tasks(*a.sc, a.N);
-            return 2 * tc_fusion_key(*a.sc) + 1;
-        }
-        *G = 0;
-        return -1;
-    };
+    auto fusion = [](const LaunchArgs &a, int *G) { return fusion_class(*a.sc, a.N, G); };
     std::vector<char> done((size_t)std::max(n, 0), 0);
     std::vector<LaunchArgs> grp;
     std::vector<int> gs;

@@ -16,6 +16,11 @@ bsr_status_t pack_data(Handle &h);
 // Launches every kernel of one bsr_spmm call on a.stream.
 cudaError_t launch_spmm(const LaunchArgs &a);
 
+// A product's fusion class at N: products with equal non-negative classes
+// (same X, N and stream) can share one grid; -1: the generic kernel, which
+// runs alone. *G receives the task size chosen for N.
+int fusion_class(const Schedule &sc, int64_t N, int *G);
+
 // Launches n products that share X, N and the stream: products whose kernels
 // share a template (xstage, or tensor-core of one dtype and R) run as one
 // grid, up to 64 at a time; generic-kernel products one after another.

@@ -88,6 +88,15 @@ def test_host_side_argument_errors(lib):
     buf = ctypes.create_string_buffer(16)
     assert lib.bsr_get_schedule(None, buf, 16) == b.BSR_ERR_INVALID_ARG
     lib.bsr_destroy(None)
+    # plans: argument checks before any CUDA call
+    plan = P()
+    assert lib.bsr_plan_create(None, None, None, None, None, 0, 0, None) == b.BSR_ERR_INVALID_ARG
+    assert lib.bsr_plan_create(None, None, None, None, None, -1, 0, ctypes.byref(plan)) == b.BSR_ERR_INVALID_ARG
+    assert lib.bsr_plan_create(None, None, None, None, None, 2, 1, ctypes.byref(plan)) == b.BSR_ERR_INVALID_ARG
+    assert plan.value is None
+    assert lib.bsr_plan_launch(None, None) == b.BSR_ERR_INVALID_ARG
+    assert lib.bsr_plan_get_order(None, None, None, 0, None) == b.BSR_ERR_INVALID_ARG
+    lib.bsr_plan_destroy(None)
 
 
 def test_parse_schedule():
