@@ -67,6 +67,8 @@ def parse():
     ap.add_argument("--workload", type=int, default=2, choices=[1, 2, 3, 4, 5],
                     help="2: the block-shape sweep (the benchmark line); 1, 3, 4, 5: a per-workload report "
                          "(one JSON line per block shape and dtype, device time against the roofline), 1 GPU")
+    ap.add_argument("--dtype", default="", help="report only this dtype (f32 or bf16; profiling runs)")
+    ap.add_argument("--weights", type=int, default=0, help="report on the first W weights only (profiling runs)")
     return ap.parse_args()
 
 
@@ -483,7 +485,12 @@ def run_report(args):
         return torch.from_numpy(a).to(dev)
 
     for dt, shape in REPORT_VARIANTS[args.workload]:
-        wl = synth.config(args.workload, dtype=dt, shape=shape)
+        if args.dtype and dt is not None and dt != args.dtype:
+            continue
+        if args.shapes and shape is not None and f"{shape[0]}x{shape[1]}" not in args.shapes.split(","):
+            continue
+        only = list(range(args.weights)) if args.weights and args.workload in (3, 4) else None
+        wl = synth.config(args.workload, dtype=dt, shape=shape, only=only)
         N, es = wl.N, (2 if wl.dtype == "bf16" else 4)
         X = dev_array(wl.make_X())
         handles, biases, flops, nbytes, roof_s = [], [], [], [], []

@@ -64,6 +64,7 @@ constexpr int NTHREADS = NWARPS * 32;
 constexpr uint64_t kDrainNs = 200000000ull;
 
 struct TcArgs {
+    CUtensorMap ymap;         // Y [N, M] in 16-column x 128-row boxes, for the epilogue's TMA stores
     int G, n_tasks;           // G: most items in a task (accumulator columns G * R)
     const int32_t *trec;      // task records: header, chunk starts, items, MMA entries
     const int32_t *trec_off;  // per task: record offset (ints)
@@ -388,27 +389,41 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
         const bool stop = ptx::named_barrier_or(1, 128, !got || !split_ok || aborted(misc));
         if (!got && et == 0) set_status(a.status, DEV_TIMEOUT);
         const int q = warp & 3;
-        const int64_t n = n0 + 32 * q + lane;
+        const int t = 32 * q + lane;   // this thread's token row in the tile
+        const int64_t n = n0 + t;
         const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16);
-        // 64 accumulator columns per round: two loads in flight, one wait
-        for (int c0 = 0; c0 < g_count * R && !stop; c0 += 64) {
+        // Every MMA has completed, so the X ring is idle: it stages Y in
+        // 16-column groups [128 tokens x 16 columns] that one thread stores by
+        // TMA (rows past N are not written), rounds of 64 accumulator columns
+        // alternating between two buffers. Split items write their fp32
+        // partials to the workspace directly.
+        constexpr uint32_t kGroupBytes = TN * 16 * sizeof(T);
+        constexpr uint32_t kRoundBytes = 4 * kGroupBytes;
+        static_assert(2 * kRoundBytes <= (F32 ? 2 : 1) * NS * kStageBytes, "Y staging exceeds the X ring");
+        int round = 0;
+        for (int c0 = 0; c0 < g_count * R && !stop; c0 += 64, round++) {
+            unsigned char *buf = base + (round & 1) * kRoundBytes;
+            if (round >= 2) {   // the stores issued from this buffer two rounds ago have read it
+                if (et == 0) ptx::bulk_wait_group_read<1>();
+                ptx::named_barrier(1, 128);
+            }
             uint32_t r0[32], r1[32];
             tmem_ld32_nowait(lane_base + c0, r0);
             if (c0 + 32 < g_count * R) tmem_ld32_nowait(lane_base + c0 + 32, r1);
             asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-            if (n >= a.N) continue;
 #pragma unroll
             for (int h = 0; h < 64; h += 16) {
                 const int col = c0 + h;
                 if (col >= g_count * R) break;
                 const int g = col / R, hr = col - g * R;
-                const int len = itab[6 * g + 5], row = itab[6 * g + 0], slot = itab[6 * g + 3];
+                const int len = itab[6 * g + 5], slot = itab[6 * g + 3];
                 float v[16];
 #pragma unroll
                 for (int j = 0; j < 16; j++) v[j] = len > 0 ? __uint_as_float(h < 32 ? r0[h + j] : r1[h - 32 + j]) : 0.f;
                 if (slot < 0) {
+                    unsigned char *row = buf + (h / 16) * kGroupBytes + t * 16 * (int)sizeof(T);
                     if constexpr (F32) {
-                        float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(a.Y) + n * a.M + (int64_t)row * R + hr);
+                        float4 *dst = reinterpret_cast<float4 *>(row);
 #pragma unroll
                         for (int j = 0; j < 4; j++)
                             dst[j] = make_float4(v[4 * j] + B_s[col + 4 * j], v[4 * j + 1] + B_s[col + 4 * j + 1],
@@ -421,17 +436,30 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                             const float hi = v[2 * j + 1] + B_s[col + 2 * j + 1];
                             pk[j] = (uint32_t)from_f32<uint16_t>(lo) | ((uint32_t)from_f32<uint16_t>(hi) << 16);
                         }
-                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<uint16_t *>(a.Y) + n * a.M + (int64_t)row * R + hr);
+                        uint4 *dst = reinterpret_cast<uint4 *>(row);
                         dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                         dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                     }
-                } else {
+                } else if (n < a.N) {
                     float4 *dst = reinterpret_cast<float4 *>(a.ws + ((int64_t)slot * a.N + n) * R + hr);
 #pragma unroll
                     for (int j = 0; j < 4; j++) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                 }
             }
+            ptx::fence_proxy_async_smem();   // the staged rows, visible to the TMA unit
+            ptx::named_barrier(1, 128);
+            if (et == 0) {
+                for (int h = 0; h < 64; h += 16) {
+                    const int col = c0 + h;
+                    if (col >= g_count * R) break;
+                    const int g = col / R, hr = col - g * R;
+                    if (itab[6 * g + 3] >= 0) continue;
+                    ptx::tma_store_2d(&a.ymap, buf + (h / 16) * kGroupBytes, itab[6 * g + 0] * R + hr, (int32_t)n0);
+                }
+                ptx::bulk_commit_group();
+            }
         }
+        if (et == 0) ptx::bulk_wait_group_all();   // no store outlives the CTA's shared memory
     }
     // ---------------- teardown: every MMA completed (the epilogue waited for
     // `done`, or the issuer never started), then free the tensor memory
@@ -445,7 +473,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
 
 template <typename T, int R>
 __global__ void __launch_bounds__(NTHREADS, 2)
-k_tc(const __grid_constant__ CUtensorMap xmap, const TcArgs a) {
+k_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ TcArgs a) {
     tc_cta<T, R>(xmap, a, blockIdx.x);
 }
 
@@ -531,6 +559,23 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
+// Y [N, M] for the epilogue's TMA stores: boxes of 16 columns x 128 token rows,
+// no swizzle (the staged rows are plain row-major).
+template <typename T>
+cudaError_t encode_y(void *Y, int64_t N, int64_t M, CUtensorMap *map) {
+    auto enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    const cuuint64_t dims[2] = {(cuuint64_t)M, (cuuint64_t)N};
+    const cuuint64_t strides[1] = {(cuuint64_t)M * sizeof(T)};
+    const cuuint32_t box[2] = {16, (cuuint32_t)TN};
+    const cuuint32_t estr[2] = {1, 1};
+    if (enc(map, sizeof(T) == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Y, dims,
+            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    return cudaSuccess;
+}
+
 uint32_t tmem_cols_for(int cols) {
     uint32_t n = 32;
     while ((int)n < cols) n <<= 1;
@@ -573,7 +618,7 @@ cudaError_t make_tc_args(const LaunchArgs &la, int G, TcArgs &a, uint32_t &smem)
     a.stall_chunk = la.stall_chunk;
     smem = a.misc_off + (4 + 6 * 32) * 4 + 1024;
     if (smem > (uint32_t)kTcMaxSmem || G * R > kTcTmemCols) return cudaErrorInvalidConfiguration;
-    return cudaSuccess;
+    return encode_y<T>(la.Y, la.N, sc.M, &a.ymap);
 }
 
 template <typename K>
