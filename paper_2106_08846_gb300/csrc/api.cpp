@@ -125,6 +125,7 @@ Schedule::~Schedule() {
         cudaFree(tc.d_rec[gi]);
         cudaFree(tc.d_rec_off[gi]);
         cudaFree(tc.d_worder[gi]);
+        cudaFree(tc.d_wstack[gi]);
     }
     cudaFree(d_indices);
 }
@@ -656,18 +657,24 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
     const Schedule &sc = *h->sched;
     int64_t split_rows = 0;   // rows split into pieces (the other reduce entries are empty rows)
     for (const Split &sp : sc.splits) split_rows += sp.nslot > 0;
+    char stacks[160] = "";   // per tensor-core task size 1, 2, 4, ...: chunks run as stacked MMAs
+    for (int gi = 0; gi < kTcTaskSizes; gi++) {
+        const size_t at = strlen(stacks);
+        snprintf(stacks + at, sizeof stacks - at, gi ? ",%" PRId64 : "%" PRId64,
+                 sc.variant == V_TC ? sc.tc.stacks[gi] : (int64_t)0);
+    }
     snprintf(buf, len,
              "variant=%s\ndtype=%s\nR=%d\nC=%d\nexec_R=%d\nexec_C=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
              "\nKB=%" PRId64 "\nnnzb=%" PRId64 "\ntokens_per_cta=%d\nthreads=%d\nsmem_bytes=%zu\n"
              "item_groups=%d\nitems=%zu\nsplit_len=%d\nsplit_rows=%" PRId64 "\nslots=%d\n"
              "empty_rows=%" PRId64 "\nmax_row_blocks=%" PRId64 "\nlaunches_per_call=%d\n"
              "structure_hash=%016" PRIx64 "\ncache_hit=%d\nschedule_reuses=%" PRId64
-             "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\n",
+             "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\ntc_stacked_chunks=%s\n",
              variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_R, sc.ex_C, sc.M, sc.K,
              sc.MB, sc.KB, sc.nnzb, sc.tn, sc.threads, sc.smem, sc.groups, sc.items.size(),
              sc.split_len, split_rows, sc.n_slots, sc.empty_rows, sc.max_row, launches_per_call(sc),
              sc.hash, (int)h->cache_hit, (int64_t)sc.reuse_count, (int64_t)g_cache_hits,
-             (int64_t)g_cache_misses);
+             (int64_t)g_cache_misses, stacks);
     return BSR_OK;
 }
 

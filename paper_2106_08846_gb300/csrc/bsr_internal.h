@@ -150,7 +150,8 @@ cudaError_t launch_tc(const LaunchArgs &a, int G);
 int tc_fusion_key(const Schedule &sc);
 // n products sharing X (equal keys, same X, N, K and stream) in one grid.
 cudaError_t launch_tc_batch(const LaunchArgs *las, const int *Gs, int n);
-cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
+cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, const int32_t *stack, int64_t n,
+                         int R, int C, void *out,
                          cudaStream_t s);
 cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t nnzb, int R, int C, uint16_t *tiles,
                             cudaStream_t s);

@@ -260,23 +260,32 @@ void plan_xstage(Schedule &sc) {
 // blocks): the items, longest first, each go to the least-loaded task that
 // still has room (ties: the lower task). Each task's record carries its items,
 // its chunk starts and its MMA entries; its block values are packed task by
-// task, chunk by chunk.
+// task, chunk by chunk. bf16 chunks in which every item of the task has one
+// block at the same column offset, all first or all not first, become stacks
+// (see tc.h): one MMA of N = g * R per K slice instead of g. An MMA of M = 128
+// and K = 16 costs one unit (about 39 SM cycles, the A tile's shared-memory
+// read) up to N of about 78 and N / 78 units above (the arithmetic).
 void plan_tc(Schedule &sc) {
     const int kc = tc_chunk_cols(sc.dt);
     const int64_t es = (int64_t)dtype_size(sc.dt);
     const int64_t nch = (sc.K + kc - 1) / kc;
     const size_t per_block = tc_block_bytes(sc.R, sc.C, sc.dt);
     const int64_t n_items = (int64_t)sc.items.size();
+    const double block_units = sc.dt == BSR_F32 ? 3.0 * sc.C / 8.0 : sc.C / 16.0;
+    const bool can_stack = sc.dt == BSR_BF16 && sc.C >= 32;
     int64_t total = 0;   // bytes of packed values over all usable G
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         const int G = kTcG[gi];
         std::vector<int32_t> &rec = sc.tc.rec[gi];
         std::vector<int32_t> &off = sc.tc.rec_off[gi];
         std::vector<int32_t> &order = sc.tc.worder[gi];
+        std::vector<int32_t> &stack = sc.tc.wstack[gi];
         rec.clear();
         off.clear();
         order.clear();
-        sc.tc.task_blocks_max[gi] = 0;
+        stack.clear();
+        sc.tc.task_cost_max[gi] = 0;
+        sc.tc.stacks[gi] = 0;
         size_t wmax = 0, imax = 0;
         const int64_t n_tasks = (n_items + G - 1) / G;
         std::vector<std::vector<int32_t>> members((size_t)n_tasks);
@@ -290,13 +299,6 @@ void plan_tc(Schedule &sc) {
                 members[(size_t)l.second].push_back((int32_t)k);
                 if ((int)members[(size_t)l.second].size() < G)
                     open.push({l.first + sc.items[(size_t)k].p1 - sc.items[(size_t)k].p0, l.second});
-                else
-                    sc.tc.task_blocks_max[gi] = std::max(sc.tc.task_blocks_max[gi],
-                                                         l.first + sc.items[(size_t)k].p1 - sc.items[(size_t)k].p0);
-            }
-            while (!open.empty()) {
-                sc.tc.task_blocks_max[gi] = std::max(sc.tc.task_blocks_max[gi], open.top().first);
-                open.pop();
             }
         }
         std::vector<std::vector<int32_t>> per_chunk((size_t)nch), src((size_t)nch);
@@ -328,6 +330,25 @@ void plan_tc(Schedule &sc) {
                 wmax = std::max(wmax, per_chunk[(size_t)c].size() * per_block);
             }
             rec[head + 4 + (size_t)nch] = n;
+            // stacks, and the task's MMA cost
+            double cost = 0.0;
+            for (int64_t c = 0; c < nch; c++) {
+                std::vector<int32_t> &pc = per_chunk[(size_t)c];
+                bool st = can_stack && g_count >= 2 && g_count * sc.R <= 256 && (int)pc.size() == g_count;
+                for (int g = 0; st && g < g_count; g++)
+                    st = ((pc[(size_t)g] >> 2) & 31) == g && (pc[(size_t)g] & 3) == (pc[0] & 3) &&
+                         ((pc[(size_t)g] >> 7) & 1) == ((pc[0] >> 7) & 1);
+                if (st) {
+                    pc[0] |= 1 << 8;
+                    sc.tc.stacks[gi]++;
+                    for (int g = 1; g < g_count; g++) pc[(size_t)g] |= 1 << 9;
+                    cost += (sc.C / 16.0) * std::max(1.0, g_count * sc.R / 78.0);
+                } else {
+                    cost += block_units * (double)pc.size();
+                }
+                for (int g = 0; g < (int)pc.size(); g++) stack.push_back(st ? (g << 16) | g_count : 1);
+            }
+            sc.tc.task_cost_max[gi] = std::max(sc.tc.task_cost_max[gi], (int64_t)std::ceil(cost));
             for (int g = 0; g < g_count; g++) {
                 const Item &it = sc.items[(size_t)mem[(size_t)g]];
                 rec[items_at + 4 * (size_t)g + 0] = it.row;
@@ -507,7 +528,8 @@ bsr_status_t build_schedule(Schedule &sc) {
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (upload(&sc.tc.d_rec[gi], sc.tc.rec[gi]) != cudaSuccess ||
             upload(&sc.tc.d_rec_off[gi], sc.tc.rec_off[gi]) != cudaSuccess ||
-            upload(&sc.tc.d_worder[gi], sc.tc.worder[gi]) != cudaSuccess) {
+            upload(&sc.tc.d_worder[gi], sc.tc.worder[gi]) != cudaSuccess ||
+            upload(&sc.tc.d_wstack[gi], sc.tc.wstack[gi]) != cudaSuccess) {
             cudaGetLastError();
             return BSR_ERR_ALLOC;
         }
@@ -543,14 +565,16 @@ bsr_status_t pack_data(Handle &h) {
                 e = reblock_tc_data((const uint16_t *)h.data, sc.d_vmap, sc.nnzb, sc.R, sc.C, (uint16_t *)tiles, 0);
             for (int gi = 0; gi < kTcTaskSizes && e == cudaSuccess; gi++)
                 if (sc.tc.w_off[gi] >= 0)
-                    e = pack_tc_data(tiles, sc.dt, sc.tc.d_worder[gi], (int64_t)sc.tc.worder[gi].size(), sc.ex_R, 64,
+                    e = pack_tc_data(tiles, sc.dt, sc.tc.d_worder[gi], sc.tc.d_wstack[gi],
+                                     (int64_t)sc.tc.worder[gi].size(), sc.ex_R, 64,
                                      (unsigned char *)h.data_packed + sc.tc.w_off[gi], 0);
             if (e == cudaSuccess) e = cudaDeviceSynchronize();
             cudaFree(tiles);
         } else {
             for (int gi = 0; gi < kTcTaskSizes && e == cudaSuccess; gi++)
                 if (sc.tc.w_off[gi] >= 0)
-                    e = pack_tc_data(h.data, sc.dt, sc.tc.d_worder[gi], (int64_t)sc.tc.worder[gi].size(), sc.R, sc.C,
+                    e = pack_tc_data(h.data, sc.dt, sc.tc.d_worder[gi], sc.tc.d_wstack[gi],
+                                     (int64_t)sc.tc.worder[gi].size(), sc.R, sc.C,
                                      (unsigned char *)h.data_packed + sc.tc.w_off[gi], 0);
         }
     } else {
@@ -603,11 +627,13 @@ int choose_tasks(const Schedule &sc, int64_t N) {
 }
 
 // Task size for the tcgen05 kernel: the G that minimises waves x (fixed CTA
-// cost + the most loaded task's MMAs), among the G whose accumulators fit
+// cost + the most loaded task's MMA cost), among the G whose accumulators fit
 // tensor memory and whose shared memory fits; a wave is every SM holding as
 // many CTAs as fit it at once. A CTA's fixed cost (tensor-memory allocation,
-// barriers, work list, first stage round trip, epilogue) is worth about
-// kOverheadMma MMAs.
+// barriers, work list, first stage round trip, epilogue: several microseconds
+// in per-CTA phase stamps) is counted as kOverheadMma MMA units, a
+// conservative weight: at 32 the model preferred five waves of two-row tasks
+// to three waves of four-row tasks on Zipf rows, measured 9% slower.
 int choose_tc_tasks(const Schedule &sc, int64_t N) {
     static const int forced = [] {
         const char *v = getenv("BSR_TC_G");
@@ -616,8 +642,7 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
     auto fits = [&](int G) { return sc.tc.w_off[tc_g_index(G)] >= 0; };   // planned and packed for G
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (forced == kTcG[gi] && fits(forced)) return forced;
-    const double kOverheadMma = 32.0;
-    const double mma_per_block = sc.dt == BSR_F32 ? 3.0 * sc.ex_C / 8.0 : sc.ex_C / 16.0;
+    const double kOverheadMma = 64.0;
     const int64_t tiles = (N + kTcTokens - 1) / kTcTokens;
     int best = 1;
     double best_cost = -1.0;
@@ -628,7 +653,7 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
         const int64_t slots = (int64_t)sc.sm_count *
                               tc_ctas_per_sm(sc.ex_R, G, sc.tc.task_wbytes[gi], sc.tc.task_ibytes[gi], sc.dt);
         const double waves = (double)((ctas + slots - 1) / slots);
-        const double cost = waves * (kOverheadMma + (double)sc.tc.task_blocks_max[gi] * mma_per_block);
+        const double cost = waves * (kOverheadMma + (double)sc.tc.task_cost_max[gi]);
         if (best_cost < 0 || cost < best_cost) {
             best_cost = cost;
             best = G;

@@ -324,6 +324,17 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                         constexpr uint32_t idesc = idesc_bf16(TN, R);
                         if (C == 16) {   // (one MMA per block: handled in batches below)
                             mma_bf16(d, ad, bd, idesc, first == 0u);
+                        } else if ((v >> 9) & 1u) {
+                            // a stack member: its rows are in its head's MMAs
+                        } else if ((v >> 8) & 1u) {
+                            // a stack head: the B operand of all g_count items' blocks,
+                            // into their adjacent accumulators
+                            const uint32_t ns = (uint32_t)(g_count * R);
+                            const uint32_t idesc_s = idesc_bf16(TN, (int)ns);
+#pragma unroll 4
+                            for (int sl = 0; sl < C / 16; sl++)
+                                mma_bf16(tmem, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * ns * 2), idesc_s,
+                                         (first == 0u) | (sl > 0));
                         } else {
 #pragma unroll 4
                             for (int sl = 0; sl < C / 16; sl++)
@@ -497,16 +508,21 @@ k_tc_batch(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ TcB
 // Block values into the MMA's B operand layout (K-major, no swizzle): for each
 // K-slice of 16 columns, 8-row x 16-byte core matrices, 128 bytes apart along
 // K and 256 bytes apart along the rows.
-// Packed block i holds stored block order[i].
+// Packed block i holds stored block order[i]; stack[i] = (g << 16) | m puts it
+// at rows g*R .. g*R+R-1 of an operand of m*R rows that starts at packed
+// block i - g (m = 1: a block of its own).
 __global__ void k_pack_tc(const uint16_t *__restrict__ data, const int32_t *__restrict__ order,
-                          uint16_t *__restrict__ out, int64_t n, int R, int C) {
+                          const int32_t *__restrict__ stack, uint16_t *__restrict__ out, int64_t n, int R, int C) {
     const int64_t total = n * R * C;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
          e += (int64_t)gridDim.x * blockDim.x) {
         const int64_t p = e / ((int64_t)R * C);
         const int rc = (int)(e - p * R * C);
-        const int n_ = rc / C, k = rc - n_ * C;
-        const int64_t dst = p * R * C + (k >> 4) * (R * 16) + (n_ >> 3) * 128 + ((k & 15) >> 3) * 64 + (n_ & 7) * 8 + (k & 7);
+        const int n0 = rc / C, k = rc - n0 * C;
+        const int sw = stack[p], g = sw >> 16, m = sw & 0xffff;
+        const int RS = m * R, n_ = g * R + n0;   // rows of the operand, this row in it
+        const int64_t dst =
+            (p - g) * R * C + (k >> 4) * (RS * 16) + (n_ >> 3) * 128 + ((k & 15) >> 3) * 64 + (n_ & 7) * 8 + (k & 7);
         out[dst] = data[(int64_t)order[p] * R * C + rc];
     }
 }
@@ -725,15 +741,16 @@ int tc_ctas_per_sm(int R, int G, size_t wbytes, size_t ibytes, bsr_dtype_t dt) {
     return std::max(1, std::min(bound, std::min(by_smem, by_tmem)));
 }
 
-cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, int64_t n, int R, int C, void *out,
-                         cudaStream_t s) {
+cudaError_t pack_tc_data(const void *data, bsr_dtype_t dt, const int32_t *order, const int32_t *stack, int64_t n,
+                         int R, int C, void *out, cudaStream_t s) {
     const int64_t total = n * R * C;
     if (total == 0) return cudaSuccess;
     const int grid = (int)std::min<int64_t>((total + 255) / 256, 1 << 20);
     if (dt == BSR_F32)
         k_pack_tc_f32<<<grid, 256, 0, s>>>(static_cast<const float *>(data), order, static_cast<float *>(out), n, R, C);
     else
-        k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), order, static_cast<uint16_t *>(out), n, R, C);
+        k_pack_tc<<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(data), order, stack, static_cast<uint16_t *>(out), n,
+                                       R, C);
     return cudaGetLastError();
 }
 

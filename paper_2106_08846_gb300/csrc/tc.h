@@ -29,14 +29,17 @@ constexpr int kTcG[kTcTaskSizes] = {1, 2, 4, 8, 16, 32};
 struct TcPlan {
     size_t task_wbytes[kTcTaskSizes] = {};   // W ring stage bytes
     size_t task_ibytes[kTcTaskSizes] = {};
-    int64_t task_blocks_max[kTcTaskSizes] = {};   // blocks of the most loaded task
+    int64_t task_cost_max[kTcTaskSizes] = {};     // MMA cost of the most loaded task (units: one N <= 64 MMA)
+    int64_t stacks[kTcTaskSizes] = {};            // stacked chunks over all tasks
     std::vector<int32_t> rec[kTcTaskSizes];       // all task records of this G
     std::vector<int32_t> rec_off[kTcTaskSizes];   // per task: offset (ints, multiple of 4)
     std::vector<int32_t> worder[kTcTaskSizes];    // per packed block: the (execution) block it holds
+    std::vector<int32_t> wstack[kTcTaskSizes];    // per packed block: (its row group in a stack << 16) | stack size
     int64_t w_off[kTcTaskSizes] = {};             // byte offset of G's packed values (-1: G not usable)
     int32_t *d_rec[kTcTaskSizes] = {};
     int32_t *d_rec_off[kTcTaskSizes] = {};
     int32_t *d_worder[kTcTaskSizes] = {};
+    int32_t *d_wstack[kTcTaskSizes] = {};
 };
 
 // A task record (int32): [ the task's first packed block, its item count g,
@@ -44,7 +47,12 @@ struct TcPlan {
 // padded to 4 | per item (row, p0, p1, slot) | one entry per MMA-block,
 // chunk by chunk, padded to 4 ]. Entry e uses packed block (first + e).
 // Entry bits: [0,2) stage column offset / 32 bytes, [2,7) item in the task,
-// 7 first block of its item.
+// 7 first block of its item, 8 stack head, 9 stack member. A stack is a chunk
+// in which every item of the task has exactly one block, at the same column
+// offset, all first or all not first (bf16 blocks of 32 or more columns): its
+// g blocks are packed as one B operand of g * R rows, and the head's MMAs
+// (N = g * R, into the accumulators of items 0..g-1, which are adjacent)
+// replace the members'.
 inline int64_t tc_pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
 bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K);

@@ -365,6 +365,32 @@ def test_small_bf16_blocks_run_as_16_row_tensor_core_tiles(R, C):
     check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M)
 
 
+@pytest.mark.parametrize("holes", [False, True])
+def test_stacked_mmas_for_dense_tile_rows(holes):
+    """Re-blocked 32x1 bf16 tiles where every tile row of a task has a tile in
+    a chunk run as one MMA over all the task's rows (a stack: N = rows x 32).
+    With holes, one tile row has no tile in chunk 2 and another starts in
+    chunk 1, so some chunks mix stacked and per-item MMAs in one task; the
+    product must match the oracle either way (many token tiles, ragged tail)."""
+    R, C, M, K, N = 32, 1, 256, 512, 5000
+    MB, KB = M // R, K // C
+    mask = synth.uniform_block_mask(90, MB, KB, int(MB * KB * 0.3))
+    if holes:
+        mask[3, 128:192] = False
+        mask[5, 0:64] = False
+    w = synth.make_weight("s", 91, M, K, R, C, "bf16", 0, mask=mask)
+    X = synth.activations(92, N, K, "bf16")
+    h, _, Y = _run(w, X)
+    s = h.schedule()
+    assert s["variant"] == "tcgen05" and s["exec_R"] == 32 and s["exec_C"] == 64
+    stacks = [int(v) for v in str(s["tc_stacked_chunks"]).split(",")]
+    assert stacks[0] == 0 and all(v > 0 for v in stacks[1:4])   # G = 1 has nothing to stack; G = 2, 4, 8 do
+    if holes:
+        assert stacks[3] < K // 64   # the task of all eight rows cannot stack chunks 0, 1 and 2
+    rows = np.concatenate([np.arange(0, 300), np.arange(N - 300, N)])
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M, rows=rows)
+
+
 def test_small_bf16_blocks_whose_rows_do_not_fill_tiles_stay_simt():
     """M not a multiple of 16 (4-row blocks, M = 260): no 16-row tiling, the
     SIMT kernel keeps the weight."""
