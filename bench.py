@@ -515,7 +515,14 @@ def run_report(args):
             flush.zero_()
             step()
         torch.cuda.synchronize()
-        K = max(1, args.steps)
+        # at least about 0.4 s of timed steps, so that the clock sampler (50 ms
+        # period) sees the region
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        K = max(1, args.steps, int(0.4 / max(e0.elapsed_time(e1) * 1e-3, 1e-6)))
         st = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
         with ClockSampler(0) as clocks:
             for k in range(K):
