@@ -391,6 +391,22 @@ def test_stacked_mmas_for_dense_tile_rows(holes):
     check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M, rows=rows)
 
 
+def test_stacked_mmas_for_32_column_bf16_blocks():
+    """Native 32x32 bf16 blocks, every block kept, K = 96: the first 64-column
+    chunk holds two blocks of every row (per-item MMAs), the second one block of
+    every row at the same offset (a stack); ragged token tail."""
+    R, C, M, K, N = 32, 32, 256, 96, 333
+    mask = np.ones((M // R, K // C), dtype=bool)
+    w = synth.make_weight("s32", 93, M, K, R, C, "bf16", 0, mask=mask)
+    X = synth.activations(94, N, K, "bf16")
+    h, _, Y = _run(w, X)
+    s = h.schedule()
+    assert s["variant"] == "tcgen05" and s["exec_C"] == 32
+    stacks = [int(v) for v in str(s["tc_stacked_chunks"]).split(",")]
+    assert stacks[0] == 0 and stacks[1] > 0
+    check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M)
+
+
 def test_small_bf16_blocks_whose_rows_do_not_fill_tiles_stay_simt():
     """M not a multiple of 16 (4-row blocks, M = 260): no 16-row tiling, the
     SIMT kernel keeps the weight."""
