@@ -16,14 +16,18 @@
 //   warp 1 (one thread)  owns the tensor memory (G * R fp32 columns, one
 //                         block row per R columns) and issues the MMAs from
 //                         the work list (per chunk, one packed entry per
-//                         block: column offset, item, first-block flag); a
+//                         block: column offset, item, first-block flag, stack
+//                         head or member); a chunk where every item has one
+//                         block is a stack: one MMA per K slice with
+//                         N = items x R over their adjacent accumulators. A
 //                         tcgen05.commit per chunk releases the stage.
 //   warps 2..5           fp32: split every landed X stage into tf32 high and
 //                         low parts (low into a twin buffer) for the issuer's
 //                         high x high + high x low + low x high; then the
 //                         epilogue: each reads its 32 TMEM lanes (tokens),
-//                         adds the bias, converts and stores Y (or an fp32
-//                         partial for a split row).
+//                         adds the bias, converts, stages 16-column groups in
+//                         the idle X ring and one thread stores them to Y by
+//                         2-D TMA (split rows write fp32 partials directly).
 //
 // Two CTAs share an SM, so that one CTA's set-up, stage round trips and
 // epilogue overlap the other's MMAs: bf16 uses a 3-stage ring, fp32 a 2-stage
