@@ -17,8 +17,15 @@
  *   Y[n, i*R + r] = bias[i*R + r]
  *                 + sum_{p = indptr[i]}^{indptr[i+1]-1} sum_{c<C} X[n, indices[p]*C + c] * data[p][r][c]
  * with X[N, K] and Y[N, M] row-major. Element types: BSR_F32 (fp32 data, X
- * and Y, fp32 accumulation, no TF32) or BSR_BF16 (bf16 data, X and Y, fp32
+ * and Y, fp32 accumulation) or BSR_BF16 (bf16 data, X and Y, fp32
  * accumulation, Y rounded to nearest even). bias is always fp32 or NULL.
+ * Plain TF32 is never used for BSR_F32. fp32 blocks of 32 or more rows with
+ * 16 or 32 columns run on the tensor cores as 3xTF32: each operand is split
+ * into a tf32 high part and a tf32 low part (the remainder) and the product is
+ * hi*hi + hi*lo + lo*hi, accumulated in fp32. The dropped lo*lo term and the
+ * rounding of the low parts leave a relative error near 2^-20 per product,
+ * inside the fp32 tolerance |dY| <= 1e-5 * (sum |x||w| + |b|). Every other
+ * fp32 shape multiplies in plain fp32 FMA.
  *
  * Conventions.
  *  - Every call returns a status; the library never aborts, prints or traps.
@@ -128,8 +135,10 @@ bsr_status_t bsr_spmm(bsr_handle_t h, const void *X, const float *bias, void *Y,
 /*
  * bsr_check_device_status -- synchronise the device and return the first
  * error a kernel of this handle recorded (BSR_ERR_TIMEOUT when a bounded
- * wait gave up, BSR_ERR_STRUCTURE when a kernel met an out-of-range index),
- * then clear it. BSR_OK if none.
+ * wait gave up), then clear it. BSR_OK if none. Structure errors are not
+ * reported here: bsr_create validates indptr/indices on the host and the
+ * kernels read only the handle's own repacked copy, built from the
+ * validated structure.
  */
 bsr_status_t bsr_check_device_status(bsr_handle_t h);
 
@@ -161,9 +170,11 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len);
  * The fp32 partial tiles of block rows that the schedule splits across CTAs
  * go to one scratch array compiled into the library, of
  * BSR_NOALLOC_SCRATCH_BYTES bytes, which every GPU that loads the library
- * holds until the process exits. A call needs slots * N * R * 4 bytes of it
- * ("slots" and "R" as reported by bsr_get_schedule); a larger call returns
- * BSR_ERR_CAPACITY and launches nothing.
+ * holds until the process exits. A call needs slots * N * exec_R * 4 bytes
+ * of it ("slots" and "exec_R" as reported by bsr_get_schedule; exec_R is the
+ * block height the kernels run, 16 for small or narrow bf16 blocks re-blocked
+ * for the tensor cores, else R); a larger call returns BSR_ERR_CAPACITY and
+ * launches nothing.
  * The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current) and keeps it: make that
  * first call before any stream capture. All calls share the one array, so

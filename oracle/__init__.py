@@ -30,8 +30,12 @@ def build(force: bool = False) -> str:
     if force or not os.path.exists(_SO) or os.path.getmtime(_SO) < max(
             os.path.getmtime(src), os.path.getmtime(os.path.join(_HERE, "ref_bsr.h"))):
         tmp = _SO + f".{os.getpid()}.tmp"
-        subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math",
-                               "-fPIC", "-shared", "-o", tmp, src, "-lm"])
+        cmd = ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared", "-o", tmp,
+               src, "-lm"]
+        try:   # OpenMP shares the float-accumulate baseline's block rows among cores
+            subprocess.check_call(cmd[:1] + ["-fopenmp"] + cmd[1:], stderr=subprocess.DEVNULL)
+        except subprocess.CalledProcessError:
+            subprocess.check_call(cmd)
         os.replace(tmp, _SO)
     return _SO
 
@@ -49,6 +53,8 @@ def _load():
         for name in ("ref_bsr_spmm", "ref_bsr_err_bound"):
             getattr(lib, name).argtypes = [I, I64, I64, I, I, P, P, P, P, P, P, I64, P]
         lib.ref_dense_linear.argtypes = [I, I64, I64, P, P, P, P, I64, P]
+        lib.ref_bsr_spmm_f32acc.argtypes = [I, I64, I64, I, I, P, P, P, P, P, P, I64, P, I]
+        lib.ref_max_threads.restype = I
         lib.ref_round_f32.argtypes = [P, P, I64]
         lib.ref_round_bf16.argtypes = [P, P, I64]
         _lib = lib
@@ -130,6 +136,30 @@ def bsr_spmm(indptr, indices, data, X, bias, M: int, rows=None) -> np.ndarray:
 def err_bound(indptr, indices, data, X, bias, M: int, rows=None) -> np.ndarray:
     """sum_k |X[n,k]| |W[m,k]| + |b[m]| for the same tokens."""
     return _apply("ref_bsr_err_bound", indptr, indices, data, X, bias, M, rows)
+
+
+def bsr_spmm_f32acc(indptr, indices, data, X, bias, M: int, rows=None, threads: int = 1) -> np.ndarray:
+    """Y = X W^T + b with a float accumulator (the timed CPU baseline), float32,
+    block rows divided among ``threads`` OpenMP threads."""
+    lib = _load()
+    data = np.ascontiguousarray(data)
+    X = np.ascontiguousarray(X)
+    if data.dtype != X.dtype:
+        raise TypeError("data and X must share a dtype")
+    _, R, C = data.shape
+    N, K = X.shape
+    r, n = _rows(rows, N)
+    out = np.zeros((n, M), dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    lib.ref_bsr_spmm_f32acc(_dtype_code(X), M, K, R, C, _ptr(np.ascontiguousarray(indptr, np.int32)),
+                            _ptr(np.ascontiguousarray(indices, np.int32)), _ptr(data), _ptr(X), _ptr(b),
+                            _ptr(r), n, _ptr(out), int(threads))
+    return out
+
+
+def max_threads() -> int:
+    """OpenMP threads the oracle library may use (1 without OpenMP)."""
+    return int(_load().ref_max_threads())
 
 
 def dense_linear(W, X, bias, rows=None) -> np.ndarray:

@@ -9,6 +9,9 @@
 
 #include <math.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 /* bfloat16 is the top half of a float: widening is a 16-bit shift. */
 static float bf16_to_float(uint16_t h) {
@@ -175,4 +178,45 @@ static uint16_t round_bf16(double x) {
 
 void ref_round_bf16(const double *in, uint16_t *out, int64_t n) {
     for (int64_t i = 0; i < n; i++) out[i] = round_bf16(in[i]);
+}
+
+/* The same product with a float accumulator (the timed CPU baseline): per
+ * output the kept blocks of row i in storage order and the columns of each
+ * block in order, each product rounded to float and added to a float sum,
+ * then + bias in float. Block rows are independent, so they are shared out
+ * among `threads` OpenMP threads; every output is still summed by one
+ * thread in the same order, so the result does not depend on the count. */
+void ref_bsr_spmm_f32acc(int dtype, int64_t M, int64_t K, int R, int C, const int32_t *indptr,
+                         const int32_t *indices, const void *data, const void *X, const float *bias,
+                         const int64_t *rows, int64_t n_rows, float *Y, int threads) {
+    int64_t MB = M / R;
+    (void)threads;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(threads > 0 ? threads : 1)
+#endif
+    for (int64_t i = 0; i < MB; i++) {
+        for (int64_t t = 0; t < n_rows; t++) {
+            int64_t n = rows ? rows[t] : t;
+            for (int r = 0; r < R; r++) {
+                float acc = 0.0f;
+                for (int64_t p = indptr[i]; p < indptr[i + 1]; p++)
+                    for (int c = 0; c < C; c++) {
+                        float x = elem_f(X, dtype, n * K + (int64_t)indices[p] * C + c);
+                        float w = elem_f(data, dtype, (p * R + r) * C + c);
+                        float prod = x * w;
+                        acc = acc + prod;
+                    }
+                int64_t m = i * R + r;
+                Y[t * M + m] = acc + (bias ? bias[m] : 0.0f);
+            }
+        }
+    }
+}
+
+int ref_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
 }

@@ -16,7 +16,8 @@
  * and the product over kept blocks is
  *   Y[n, i*R + r] = b[i*R + r] + sum_{p in row i} sum_c X[n, indices[p]*C + c] * data[p][r][c].
  *
- * Everything accumulates in double. Element types: ORACLE_F32 (float) or
+ * Everything accumulates in double (ref_bsr_spmm_f32acc: float, the timed
+ * CPU baseline). Element types: ORACLE_F32 (float) or
  * ORACLE_BF16 (uint16 bfloat16 bit patterns, widened exactly).
  */
 #ifndef REF_BSR_H
@@ -60,6 +61,17 @@ void ref_bsr_err_bound(int dtype, int64_t M, int64_t K, int R, int C, const int3
 /* Dense Y[t, m] = sum_k X[n_t, k] W[m, k] (k ascending, double) + bias[m]. */
 void ref_dense_linear(int dtype, int64_t M, int64_t K, const void *W, const void *X,
                       const float *bias, const int64_t *rows, int64_t n_rows, double *Y);
+
+/* As ref_bsr_spmm with a float accumulator, the timed CPU baseline: the
+ * same order per output, every product and partial sum rounded to float,
+ * then + bias[m] in float. Block rows are divided among `threads` OpenMP
+ * threads (one thread per output, so results do not depend on the count). */
+void ref_bsr_spmm_f32acc(int dtype, int64_t M, int64_t K, int R, int C, const int32_t *indptr,
+                         const int32_t *indices, const void *data, const void *X, const float *bias,
+                         const int64_t *rows, int64_t n_rows, float *Y, int threads);
+
+/* Threads the library may use (1 when built without OpenMP). */
+int ref_max_threads(void);
 
 /* Round double results to the output element type: float (round to nearest
  * even), or bfloat16 bits (round to nearest even, overflow to infinity). */

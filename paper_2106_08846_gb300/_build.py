@@ -19,6 +19,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libbsr_gb300.so")
+PROBE_SRC = os.path.join(PKG, "probe", "fp32_peak.cu")
+PROBE_LIB = os.path.join(PKG, "libbsr_probe.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-I", INCLUDE, "-I", CSRC]
@@ -59,15 +61,31 @@ def _compile(src: str, extra: List[str]) -> str:
     return obj
 
 
+def build_probe(force: bool = False) -> str:
+    """The benchmark's FP32 FMA peak probe (libbsr_probe.so, not part of the C ABI)."""
+    if force or _stale(PROBE_LIB, [PROBE_SRC]):
+        tmp = PROBE_LIB + f".{os.getpid()}.tmp"
+        cmd = [nvcc()] + ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-shared", PROBE_SRC,
+                                 "-o", tmp, "-lcudart_static"]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed for {PROBE_SRC}:\n{' '.join(cmd)}\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, PROBE_LIB)
+    return PROBE_LIB
+
+
 def build(force: bool = False, extra: List[str] = (), jobs: int = 0) -> str:
-    """Compile every unit under csrc/ and link libbsr_gb300.so; returns its path."""
+    """Compile every unit under csrc/ and link libbsr_gb300.so (and the peak
+    probe, libbsr_probe.so); returns the library's path."""
     os.makedirs(OBJDIR, exist_ok=True)
     if force:
         for o in glob.glob(os.path.join(OBJDIR, "*.o")):
             os.remove(o)
     srcs = sources()
-    with cf.ThreadPoolExecutor(max_workers=jobs or min(len(srcs), os.cpu_count() or 4)) as ex:
+    with cf.ThreadPoolExecutor(max_workers=jobs or min(len(srcs) + 1, os.cpu_count() or 4)) as ex:
+        probe = ex.submit(build_probe, force)
         objs = list(ex.map(lambda s: _compile(s, list(extra)), srcs))
+        probe.result()
     if _stale(LIB, objs):
         tmp = LIB + f".{os.getpid()}.tmp"
         cmd = [nvcc()] + ARCH + ["-shared", "-o", tmp] + objs + ["-lcudart_static"]

@@ -648,7 +648,6 @@ bsr_status_t bsr_check_device_status(bsr_handle_t h) {
         return BSR_ERR_CUDA;
     }
     if (v == DEV_TIMEOUT) return BSR_ERR_TIMEOUT;
-    if (v == DEV_BAD_INDEX) return BSR_ERR_STRUCTURE;
     return BSR_OK;
 }
 

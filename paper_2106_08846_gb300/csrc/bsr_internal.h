@@ -38,7 +38,7 @@ enum Variant : int {
 const char *variant_name(int v);
 
 // Device-side status word values (first error wins).
-enum : int { DEV_OK = 0, DEV_TIMEOUT = 1, DEV_BAD_INDEX = 2 };
+enum : int { DEV_OK = 0, DEV_TIMEOUT = 1 };
 
 // Everything derived from (device, dtype, R, C, M, K, indptr, indices): shared
 // between handles whose structure is identical.

@@ -86,10 +86,10 @@ cudaError_t launch_generic(const LaunchArgs &a) {
     const int64_t work = (int64_t)n_items * n_tiles;
     const int grid = (int)std::min<int64_t>(work, 1 << 24);
     if (sc.dt == BSR_F32)
-        return launch_kernel(k_generic<float>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Item *)sc.d_items,
+        return launch_kernel(k_generic<float>, dim3(grid), dim3(256), 0, a.stream, (const Item *)sc.d_items,
                              n_items, (const int32_t *)sc.d_indices, (const float *)a.data, (const float *)a.X,
                              a.bias, (float *)a.Y, a.ws, a.N, sc.K, sc.M, sc.R, sc.C, tn, n_tiles);
-    return launch_kernel(k_generic<uint16_t>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Item *)sc.d_items,
+    return launch_kernel(k_generic<uint16_t>, dim3(grid), dim3(256), 0, a.stream, (const Item *)sc.d_items,
                          n_items, (const int32_t *)sc.d_indices, (const uint16_t *)a.data, (const uint16_t *)a.X,
                          a.bias, (uint16_t *)a.Y, a.ws, a.N, sc.K, sc.M, sc.R, sc.C, tn, n_tiles);
 }
@@ -103,9 +103,9 @@ cudaError_t launch_reduce(const LaunchArgs &a) {
     const int64_t n_tiles = (a.N + tn - 1) / tn;
     const int grid = (int)std::min<int64_t>((int64_t)n_splits * n_tiles, 1 << 20);
     if (sc.dt == BSR_F32)
-        return launch_kernel(k_reduce<float>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
+        return launch_kernel(k_reduce<float>, dim3(grid), dim3(256), 0, a.stream, (const Split *)sc.d_splits,
                              n_splits, (const float *)a.ws, a.bias, (float *)a.Y, a.N, sc.M, R, tn, n_tiles);
-    return launch_kernel(k_reduce<uint16_t>, dim3(grid), dim3(256), 0, a.stream, 1u, (const Split *)sc.d_splits,
+    return launch_kernel(k_reduce<uint16_t>, dim3(grid), dim3(256), 0, a.stream, (const Split *)sc.d_splits,
                          n_splits, (const float *)a.ws, a.bias, (uint16_t *)a.Y, a.N, sc.M, R, tn, n_tiles);
 }
 

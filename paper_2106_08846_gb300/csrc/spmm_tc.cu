@@ -684,7 +684,7 @@ cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n) {
         if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
         const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
         if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-        return launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem, las[0].stream, 1u, map, a);
+        return launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem, las[0].stream, map, a);
     }
     if (n > kTcBatchMax) return cudaErrorInvalidValue;
     TcBatch b;
@@ -708,7 +708,7 @@ cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n) {
     cudaError_t e = allow_smem(k_tc_batch<T, R>, attr_set_b);
     if (e != cudaSuccess) return e;
     if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
-    return launch_kernel(k_tc_batch<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem_max, las[0].stream, 1u, map, b);
+    return launch_kernel(k_tc_batch<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem_max, las[0].stream, map, b);
 }
 
 }  // namespace

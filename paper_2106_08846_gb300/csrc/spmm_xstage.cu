@@ -7,14 +7,12 @@
 // inner product over the kept blocks is FP32-FMA bound, so the design goal
 // is a high share of packed FMAs among the issued instructions:
 //
-//  * The CL CTAs of a thread-block cluster share one token tile (different
-//    tasks). X[n0 : n0+64, k0 : k0+128] chunks stream through a 3-stage
-//    shared-memory ring: each CTA's producer thread loads a 64/CL-row slice
-//    of the chunk with a 2-D TMA multicast (128-byte swizzle, rows = tokens)
-//    into the same stage of every CTA of the cluster. A stage's "full"
-//    mbarrier counts the bytes of all slices; every consumer warp waits for
-//    every chunk in order, processes all of its blocks that fall in it, and
-//    releases the stage on the "empty" mbarrier of every CTA in the cluster.
+//  * X[n0 : n0+64, k0 : k0+128] chunks stream through a 3-stage
+//    shared-memory ring: the producer thread loads each chunk with 2-D TMA
+//    tile loads (128-byte swizzle, rows = tokens) into its own stage. A
+//    stage's "full" mbarrier counts the chunk's bytes; every consumer warp
+//    waits for every chunk in order, processes all of its blocks that fall
+//    in it, and releases the stage on the stage's "empty" mbarrier.
 //  * Per task, the producer bulk-copies one blob (built at create time):
 //    the item table, the items' records -- each block's X offset inside a
 //    stage (1-column blocks) or block column, and the first block of every
@@ -38,8 +36,7 @@
 //    touched only after that wait).
 //
 // Every wait is bounded by the global timer; a timeout sets the device
-// status word, stops the CTA's pipeline and drains its TMA loads. A cluster
-// barrier closes the kernel: no CTA leaves while another may still signal it.
+// status word, stops the CTA's pipeline and drains its TMA loads.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -485,7 +482,7 @@ __device__ __forceinline__ void output_pass(const XsArgs &a, const Shared &sh, c
 // whole items, with one register tile each, and needs no tree.
 template <typename T, int TR, int NRG, int CT, int RW, int NW>
 __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int64_t n0, int task,
-                                         int g_count, uint32_t CL, int warp, int lane) {
+                                         int g_count, int warp, int lane) {
     using St = Stage<T>;
     constexpr int R = TR * NRG;
     const int C = CT ? CT : a.C;
@@ -541,11 +538,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
                 }
             }
             __syncwarp();
-            if (CL == 1) {
-                if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
-            } else if (lane < (int)CL) {
-                ptx::mbar_arrive_cluster(ptx::mapa(ptx::smem_addr(&sh.empty[c % NS]), lane));
-            }
+            if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
         }
         if (!ok && lane == 0) {
             set_status(a.status, DEV_TIMEOUT);
@@ -581,11 +574,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
         if (has_item)
             item_chunk<T, TR, NRG, CT>(acc, lane_base + (c % NS) * St::kBytes, idx, cb, wbase, c, piece, S, ks, tgx, C);
         __syncwarp();
-        if (CL == 1) {
-            if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
-        } else if (lane < (int)CL) {
-            ptx::mbar_arrive_cluster(ptx::mapa(ptx::smem_addr(&sh.empty[c % NS]), lane));
-        }
+        if (lane == 0) ptx::mbar_arrive(&sh.empty[c % NS]);
     }
     if (!ok && lane == 0) {
         set_status(a.status, DEV_TIMEOUT);
@@ -611,7 +600,7 @@ __device__ __forceinline__ void consumer(const XsArgs &a, const Shared &sh, int6
 }
 
 // One CTA of the product described by `a`; `cta` is the CTA's index within
-// that product's grid (clusters of CL consecutive CTAs).
+// that product's grid (token tiles fastest, then tasks).
 template <typename T, int TR, int NRG, int CT, int RW, int NW>
 __device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs &a, unsigned cta) {
     using St = Stage<T>;
@@ -629,13 +618,10 @@ __device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs
 
     ptx::pdl_launch_dependents();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // clusters in tile-fastest order (concurrent clusters spread over tiles);
-    // the CTAs of a cluster take consecutive tasks of the same tile
-    const uint32_t CL = ptx::cluster_nctarank(), rank = ptx::cluster_ctarank();
+    // tile-fastest order: CTAs running at the same time spread over tiles
     const int64_t n_tiles = (a.N + TN - 1) / TN;
-    const int64_t cluster_id = cta / CL;
-    const int task = (int)(cluster_id / n_tiles) * (int)CL + (int)rank;
-    const int64_t n0 = (cluster_id % n_tiles) * TN;
+    const int task = (int)(cta / n_tiles);
+    const int64_t n0 = (int64_t)(cta % n_tiles) * TN;
     const int item_first = task * a.G;
     const int g_count = task < a.n_tasks ? min(a.G, a.n_items - item_first) : 0;
     const int nch = a.nchunks;
@@ -643,14 +629,13 @@ __device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; s++) {
             ptx::mbar_init(&sh.full[s], 1);
-            ptx::mbar_init(&sh.empty[s], NW * CL);
+            ptx::mbar_init(&sh.empty[s], NW);
         }
         ptx::mbar_init(sh.wbar, 1);
         sh.misc[0] = 0;
         ptx::fence_barrier_init();
     }
-    // every CTA's barriers exist before any multicast or remote arrive
-    if (CL == 1) __syncthreads(); else ptx::cluster_sync();
+    __syncthreads();   // the barriers exist before any copy or arrive
 
     if (warp == NW) {
         // ---------------- producer: block values by bulk copy, then X chunks
@@ -661,14 +646,12 @@ __device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs
             }
             ptx::prefetch_tensormap(&xmap);
             ptx::pdl_wait();   // X may be an earlier kernel's output
-            const int rows = TN / (int)CL;                       // this CTA's slice of every chunk
-            const uint16_t mask = (uint16_t)((1u << CL) - 1u);
             int c = 0;
             bool ok = true;
             for (; c < nch; c++) {
                 const int s = c % NS;
-                // the stage is free once every consumer warp of the cluster released it
-                if (c >= NS && !ptx::mbar_wait_cluster_bounded(&sh.empty[s], ((c / NS) - 1) & 1, a.wait_ns)) {
+                // the stage is free once every consumer warp released it
+                if (c >= NS && !ptx::mbar_wait_bounded(&sh.empty[s], ((c / NS) - 1) & 1, a.wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -677,9 +660,8 @@ __device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs
                 ptx::mbar_arrive_expect_tx(&sh.full[s], St::kBytes);
 #pragma unroll
                 for (int b = 0; b < St::kBoxes; b++)
-                    ptx::tma_load_2d_multicast(sh.base + s * St::kBytes + b * St::kBoxBytes + rank * rows * 128,
-                                               &xmap, c * KC + b * St::kBoxCols, (int32_t)(n0 + rank * rows),
-                                               &sh.full[s], mask);
+                    ptx::tma_load_2d(sh.base + s * St::kBytes + b * St::kBoxBytes, &xmap, c * KC + b * St::kBoxCols,
+                                     (int32_t)n0, &sh.full[s]);
             }
             if (!ok) {
                 set_status(a.status, DEV_TIMEOUT);
@@ -693,9 +675,8 @@ __device__ __forceinline__ void xstage_cta(const CUtensorMap &xmap, const XsArgs
         }
         __syncwarp();
     } else {
-        consumer<T, TR, NRG, CT, RW, NW>(a, sh, n0, task, g_count, CL, warp, lane);
+        consumer<T, TR, NRG, CT, RW, NW>(a, sh, n0, task, g_count, warp, lane);
     }
-    if (CL > 1) ptx::cluster_sync();   // no CTA leaves while a peer may still arrive on its barriers
 }
 
 template <typename T, int TR, int NRG, int CT, int RW, int NW>
@@ -704,7 +685,7 @@ k_xstage(const __grid_constant__ CUtensorMap xmap, const XsArgs a) {
     xstage_cta<T, TR, NRG, CT, RW, NW>(xmap, a, blockIdx.x);
 }
 
-// Several products sharing X in one grid (no clusters): product h owns CTAs
+// Several products sharing X in one grid: product h owns CTAs
 // start[h] .. start[h+1]-1, with its own arguments and shared-memory layout
 // (the launch gives every CTA the largest).
 struct XsBatch {
@@ -773,49 +754,6 @@ size_t region_bytes(bsr_dtype_t dt, int R) {
     return (std::max(ring, part) + 1023) & ~size_t(1023);
 }
 
-// Whether clusters of CL CTAs with `smem` bytes each can be resident at all
-// (cached per kernel, cluster size, shared-memory size and device).
-bool cluster_fits(const void *func, int CL, uint32_t smem, int dev, int threads) {
-    struct Entry {
-        const void *func;
-        int CL, dev;
-        uint32_t smem;
-        bool ok;
-    };
-    static std::mutex mu;
-    static std::vector<Entry> cache;
-    std::lock_guard<std::mutex> lk(mu);
-    for (const Entry &e : cache)
-        if (e.func == func && e.CL == CL && e.smem == smem && e.dev == dev) return e.ok;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)CL);
-    cfg.blockDim = dim3((unsigned)threads);
-    cfg.dynamicSmemBytes = smem;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)CL;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    const bool ok = cudaOccupancyMaxActiveClusters(&n, func, &cfg) == cudaSuccess && n > 0;
-    cudaGetLastError();
-    cache.push_back({func, CL, dev, smem, ok});
-    return ok;
-}
-
-// CTAs per cluster. Multicast only pays where L2 bandwidth, not latency,
-// limits the X stream, so it is opt-in (BSR_XS_CL = 2, 4 or 8).
-int choose_cluster(int n_tasks) {
-    static const int forced = [] {
-        const char *v = getenv("BSR_XS_CL");
-        return v ? atoi(v) : 0;
-    }();
-    if (forced == 2 || forced == 4 || forced == 8) return std::min(forced, std::max(1, n_tasks));
-    return 1;
-}
-
 // Kernel arguments and dynamic shared-memory bytes of one product at task
 // size G (nothing to launch: n_items == 0 or N == 0 leaves smem = 0).
 template <int NW>
@@ -853,15 +791,15 @@ cudaError_t make_args(const LaunchArgs &la, const XsPlan &pl, int G, XsArgs &a, 
     return smem > kXsMaxSmem ? cudaErrorInvalidConfiguration : cudaSuccess;
 }
 
-// The 2-D tensor map of X [N, K] for the ring's boxes (rows per box: TN / CL).
+// The 2-D tensor map of X [N, K] for the ring's boxes (TN token rows each).
 template <typename T>
-cudaError_t encode_x(const void *X, int64_t N, int64_t K, int CL, CUtensorMap *map) {
+cudaError_t encode_x(const void *X, int64_t N, int64_t K, CUtensorMap *map) {
     auto enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
     const size_t es = sizeof(T);
     const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)N};
     const cuuint64_t strides[1] = {(cuuint64_t)K * es};
-    const cuuint32_t box[2] = {(cuuint32_t)Stage<T>::kBoxCols, (cuuint32_t)(TN / CL)};
+    const cuuint32_t box[2] = {(cuuint32_t)Stage<T>::kBoxCols, (cuuint32_t)TN};
     const cuuint32_t estr[2] = {1, 1};
     CUresult r = enc(map, es == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                      const_cast<void *>(X), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -882,7 +820,7 @@ cudaError_t allow_smem(K kernel, std::atomic<uint64_t> &done) {
 }
 
 // n products sharing X (same dtype, K, N, block shape and template); n == 1
-// is the plain launch (clusters allowed), n > 1 one fused grid.
+// is the plain launch, n > 1 one fused grid.
 template <typename T, int TR, int NRG, int CT, int RW, int NW>
 cudaError_t launch_t(const LaunchArgs *las, const int *Gs, int n, const XsPlan *const *pls) {
     constexpr int NTHREADS = (NW + 1) * 32;
@@ -895,21 +833,12 @@ cudaError_t launch_t(const LaunchArgs *las, const int *Gs, int n, const XsPlan *
         if (e != cudaSuccess || smem == 0) return e;
         static std::atomic<uint64_t> attr_set{0};   // per instantiation, one bit per device
         if ((e = allow_smem(k_xstage<T, TR, NRG, CT, RW, NW>, attr_set)) != cudaSuccess) return e;
-        int dev = 0;
-        cudaGetDevice(&dev);
-        for (int CL = choose_cluster(a.n_tasks); CL >= 1; CL >>= 1) {
-            if (CL > 1 && !cluster_fits(reinterpret_cast<const void *>(k_xstage<T, TR, NRG, CT, RW, NW>), CL, smem,
-                                        dev, NTHREADS))
-                continue;
-            const int64_t n_groups = (a.n_tasks + CL - 1) / CL;
-            const int64_t grid = n_tiles * n_groups * CL;   // cluster-major, tile-fastest
-            if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-            CUtensorMap map;
-            if ((e = encode_x<T>(la.X, la.N, la.sc->K, CL, &map)) != cudaSuccess) return e;
-            return launch_kernel(k_xstage<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem,
-                                 la.stream, (unsigned)CL, map, a);
-        }
-        return cudaErrorInvalidConfiguration;
+        const int64_t grid = n_tiles * a.n_tasks;   // task-major, tile-fastest
+        if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
+        CUtensorMap map;
+        if ((e = encode_x<T>(la.X, la.N, la.sc->K, &map)) != cudaSuccess) return e;
+        return launch_kernel(k_xstage<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem, la.stream,
+                             map, a);
     }
     if (n > kXsBatchMax) return cudaErrorInvalidValue;
     XsBatch b;
@@ -933,9 +862,9 @@ cudaError_t launch_t(const LaunchArgs *las, const int *Gs, int n, const XsPlan *
     cudaError_t e = allow_smem(k_xstage_batch<T, TR, NRG, CT, RW, NW>, attr_set_b);
     if (e != cudaSuccess) return e;
     CUtensorMap map;
-    if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, 1, &map)) != cudaSuccess) return e;
+    if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
     return launch_kernel(k_xstage_batch<T, TR, NRG, CT, RW, NW>, dim3((unsigned)grid), dim3(NTHREADS), smem_max,
-                         las[0].stream, 1u, map, b);
+                         las[0].stream, map, b);
 }
 
 // One-row blocks: kXsConsumerWarpsR1 consumer warps (their register tiles

@@ -57,3 +57,21 @@ def test_single_rank_max_is_identity():
     import bench
     assert bench.max_over_ranks(3.25, 1) == 3.25
     bench.barrier(1)   # no process group needed
+
+
+def test_reference_arm_prints_one_line(capsys):
+    # the reference arm (the oracle on the host cores) on the headline
+    # workload's config, at one step: one JSON line with the contract's keys
+    import json
+
+    import bench
+
+    class A:
+        steps, warmup, gpus = 1, 0, 1
+    bench.run_reference(A(), 1, 0)
+    lines = [ln for ln in capsys.readouterr().out.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["unit"] == "GFLOP/s" and d["value"] > 0
+    assert d["higher_is_better"] is True and d["cpu_baseline"]["cores"] >= 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["config"]["workload"] == bench.WORKLOAD

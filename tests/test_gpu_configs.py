@@ -1,7 +1,10 @@
 """The five benchmark workloads at full size, through the C ABI in the launch
-configuration the benchmark uses. The oracle checks a sample of tokens one by
-one (first, last and seeded random ones) for every weight; the builder is
-checked bit for bit against the oracle for every weight."""
+configuration the benchmark uses. For every weight the builder is checked bit
+for bit against the oracle, and the product on a sample of tokens (first,
+last and seeded random ones) plus one whole 128-token tile from the middle of
+N (a tile of the full-size launch: its CTA count, task sizes and waves differ
+from the small tests'); at least one weight of every kernel configuration the
+workloads launch is checked on every token."""
 import numpy as np
 import pytest
 import torch
@@ -18,7 +21,13 @@ def _sample_rows(N, k, seed):
     return np.unique(np.concatenate([[0, N - 1], rng.choice(N, size=min(k, N), replace=False)]))
 
 
-def _check_workload(wl, sample=12):
+def _middle_tile(N, tile=128):
+    start = max(0, (N // 2) // tile * tile)
+    return np.arange(start, min(N, start + tile))
+
+
+def _check_workload(wl, sample=12, full=()):
+    """`full`: indices of weights checked on every token."""
     import paper_2106_08846_gb300 as bsr
     X = wl.make_X()
     Xd = to_dev(X)
@@ -31,7 +40,10 @@ def _check_workload(wl, sample=12):
         torch.cuda.synchronize()
         assert h.check_device_status() == 0
         Yh = to_host(Y)
-        rows = _sample_rows(wl.N, sample, 17 + i)
+        if i in full:
+            rows = None
+        else:
+            rows = np.union1d(_sample_rows(wl.N, sample, 17 + i), _middle_tile(wl.N))
         check_product(Yh, ref, X, w.bias, w.M, rows=rows)
         h.destroy()
 
@@ -42,22 +54,28 @@ def test_config1_bert_base_single_weight():
 
 
 def test_config2_block_shape_sweep():
-    _check_workload(synth.config(2), sample=24)
+    wl = synth.config(2)
+    _check_workload(wl, full=range(len(wl.weights)))   # every shape, every token
 
 
 def test_config3_bert_base_projection_set():
-    # all 48 weights built and run; the oracle samples 4 tokens of each
-    _check_workload(synth.config(3), sample=4)
+    # all 48 weights built and run; the oracle checks 4 sampled tokens and a
+    # middle tile of each, and every token of one weight per sparsity level
+    wl = synth.config(3)
+    sp = synth.sweep_sparsities(48)
+    full = {sp.index(s) for s in set(sp)}
+    _check_workload(wl, sample=4, full=full)
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("shape", [(32, 1), (16, 16)])
 def test_config4_bert_large(dtype, shape):
-    # first and last layer's Q/K/V/O (8 of 96 weights) at the full 16384 tokens
+    # first and last layer's Q/K/V/O (8 of 96 weights) at the full 16384
+    # tokens; the first on every token
     wl = synth.config(4, dtype=dtype, shape=shape, only=[0, 1, 2, 3, 92, 93, 94, 95])
-    _check_workload(wl, sample=4)
+    _check_workload(wl, sample=4, full={0})
 
 
 @pytest.mark.parametrize("shape", [(32, 1), (16, 16)])
 def test_config5_zipf_rows(shape):
-    _check_workload(synth.config(5, shape=shape), sample=6)
+    _check_workload(synth.config(5, shape=shape), full={0})

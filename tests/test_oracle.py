@@ -283,3 +283,73 @@ def test_round_bf16_brute_force_on_doubles():
         dlo, dhi = xi - vals[lo], vals[hi] - xi
         want = lo if dlo < dhi else hi if dhi < dlo else (lo if lo % 2 == 0 else hi)
         assert gi == want, (xi, gi, want)
+
+
+# ---------------------------------------------------------------- float-accumulate variant (timed baseline)
+
+@pytest.mark.parametrize("R,C", [(32, 1), (16, 16), (1, 1), (1, 32), (3, 2)])
+def test_f32acc_exact_on_dyadic_inputs(R, C):
+    # small integers scaled by powers of two: every product and partial sum
+    # is exact in float, so the float-accumulated product must equal numpy's
+    # float64 matmul of the densified weight exactly (non-square: a
+    # transposed operand fails)
+    M, K, N = 96, 160, 7
+    rng = np.random.default_rng(R * 31 + C)
+    MB, KB = M // R, K // C
+    mask = rng.random((MB, KB)) < 0.35
+    W = (rng.integers(-8, 9, size=(M, K)) / 8.0).astype(np.float32)
+    W *= np.kron(mask, np.ones((R, C))).astype(np.float32)
+    W[W == 0] = 0.0
+    X = rng.integers(-16, 17, size=(N, K)).astype(np.float32)
+    b = (rng.integers(-4, 5, size=M) / 4.0).astype(np.float32)
+    ref = sp.bsr_matrix(W, blocksize=(R, C))
+    ref.sort_indices()
+    bsr = oracle.bsr_from_dense(W, R, C)
+    Y = oracle.bsr_spmm_f32acc(*bsr, X, b, M)
+    want = X.astype(np.float64) @ W.astype(np.float64).T + b
+    assert Y.dtype == np.float32
+    assert np.array_equal(Y.astype(np.float64), want)
+
+
+def test_f32acc_within_rounding_bound():
+    # n float additions of rounded products: |error| <= gamma_(n+1) * sum |x||w|
+    # (Higham, Accuracy and Stability of Numerical Algorithms, Sec. 3.1),
+    # u = 2^-24, n = terms per output (+1 for the bias)
+    R, C, M, K, N = 8, 4, 64, 256, 19
+    W, _ = _block_weight(M, K, R, C, 0.4, 901)
+    X = synth.activations(902, N, K, "f32")
+    b = synth.normal(903, synth.STREAM_BIAS, M, 0.02)
+    bsr = oracle.bsr_from_dense(W, R, C)
+    Y = oracle.bsr_spmm_f32acc(*bsr, X, b, M).astype(np.float64)
+    exact = X.astype(np.float64) @ W.astype(np.float64).T + b
+    E = np.abs(X.astype(np.float64)) @ np.abs(W.astype(np.float64)).T + np.abs(b)
+    terms = np.diff(bsr[0]).max() * C + 1
+    u = 2.0 ** -24
+    gamma = (terms + 1) * u / (1 - (terms + 1) * u)
+    assert np.all(np.abs(Y - exact) <= gamma * E)
+    # and it is not the float64 result rounded once: float accumulation differs somewhere
+    assert not np.array_equal(Y, exact.astype(np.float32).astype(np.float64))
+
+
+def test_f32acc_independent_of_threads_and_tokens():
+    R, C, M, K, N = 16, 1, 128, 96, 33
+    W, _ = _block_weight(M, K, R, C, 0.5, 911)
+    X = synth.activations(912, N, K, "f32")
+    b = np.linspace(-0.1, 0.1, M).astype(np.float32)
+    bsr = oracle.bsr_from_dense(W, R, C)
+    Y1 = oracle.bsr_spmm_f32acc(*bsr, X, b, M, threads=1)
+    for t in (2, 3, 8):
+        assert np.array_equal(Y1, oracle.bsr_spmm_f32acc(*bsr, X, b, M, threads=t))
+    rows = [32, 0, 17]
+    assert np.array_equal(Y1[rows], oracle.bsr_spmm_f32acc(*bsr, X, b, M, rows=rows, threads=4))
+
+
+def test_f32acc_full_sparsity_gives_bias_bf16():
+    M, K, R, C = 32, 64, 16, 16
+    W = np.zeros((M, K), dtype=np.uint16)
+    X = synth.to_bf16_bits(synth.activations(921, 5, K, "f32"))
+    b = np.linspace(-1, 1, M).astype(np.float32)
+    bsr = oracle.bsr_from_dense(W, R, C)
+    assert bsr[0][-1] == 0
+    Y = oracle.bsr_spmm_f32acc(*bsr, X, b, M, threads=2)
+    assert np.array_equal(Y, np.broadcast_to(b, (5, M)))
