@@ -78,6 +78,10 @@ def parse(argv=None):
     ap.add_argument("--dtype", default="", help="report only this dtype (f32 or bf16)")
     ap.add_argument("--shapes", default="", help="comma-separated subset of block shapes, e.g. 32x1,16x16")
     ap.add_argument("--weights", type=int, default=0, help="use the first W weights of workloads 3 and 4 only")
+    ap.add_argument("--min-seconds", type=float, default=MIN_TIMED_S,
+                    help="time at least this long (0: exactly --steps steps; profiling runs)")
+    ap.add_argument("--no-probe", action="store_true",
+                    help="skip the FP32 peak probe and use the derived peak (profiling runs)")
     return ap.parse_args(argv)
 
 
@@ -227,6 +231,13 @@ def dev_array(a, dev):
 
 
 # ------------------------------------------------------------------ FP32 FMA peak
+
+def derived_fp32_peak(dev, pk):
+    import torch
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    t = sms * 128 * 2 * float(pk.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+    return {"fma_f32x2_sustained": t, "source": f"derived: {sms} SMs x 128 FP32 lanes x 2 x max clock (not measured)"}
+
 
 def fp32_peak(dev, stream, sustained_s=1.5):
     """Measured FP32 multiply-add rate (TFLOP/s) of the probe kernel on every
@@ -413,7 +424,7 @@ def kernel_key(sc, w):
 
 def pipe_peak(sc, dtype, pk, fp32_tflops):
     """(peak FLOP/s, description) of the pipe that bounds this kernel's arithmetic."""
-    if sc["variant"] == "tc":
+    if sc["variant"] == "tcgen05":
         bf16 = float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"])) * 1e12
         if dtype == "bf16":
             return bf16, f"bf16 tensor, sustained ({pk['source']})"
@@ -466,7 +477,8 @@ def enqueue_seconds(prod, stream):
     return s
 
 
-def measure(prod, K_req, warmup, stream, flush, pk, fp32_tflops, hbm, world=1, clocks_index=None):
+def measure(prod, K_req, warmup, stream, flush, pk, fp32_tflops, hbm, world=1, clocks_index=None,
+            min_s=MIN_TIMED_S):
     """Step times (flushed and hot L2), per-kernel roofline and the step roofline."""
     import torch
     for _ in range(max(warmup, 3)):
@@ -474,7 +486,7 @@ def measure(prod, K_req, warmup, stream, flush, pk, fp32_tflops, hbm, world=1, c
         prod.step(stream)
     torch.cuda.synchronize()
     one = timed_steps(lambda: prod.step(stream), 1, stream, flush)[0] * 1e-3
-    K = max(K_req, int(math.ceil(MIN_TIMED_S / max(one, 1e-6))))
+    K = max(K_req, int(math.ceil(min_s / max(one, 1e-6))))
     enq = enqueue_seconds(prod, stream)
     hold = min(enq * K * 1.5 + 0.01, 2.0)
     barrier(world)
@@ -526,7 +538,7 @@ def kernel_roofline(d, hbm):
         r = {"bound": "hbm", "achieved": nbytes / t / 1e9, "peak": hbm / 1e9, "unit": "GB/s",
              "peak_source": "HBM copy bandwidth, MEASURED_PEAKS.json"}
     else:
-        r = {"bound": "alu" if sc["variant"] != "tc" else "tensor", "achieved": flops / t / 1e12,
+        r = {"bound": "alu" if sc["variant"] != "tcgen05" else "tensor", "achieved": flops / t / 1e12,
              "peak": d["peak"] / 1e12, "unit": "TFLOP/s", "peak_source": d["peak_desc"]}
     r["frac"] = r["achieved"] / r["peak"]
     r["traffic"] = profiled_traffic(kernel_key(sc, w) + f"_{w.M}x{w.K}")
@@ -626,7 +638,7 @@ def run_ours(args, world, rank, local):
     hbm = float(pk["hbm_gbs"]) * 1e9
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
 
-    fp32 = fp32_peak(dev, stream)
+    fp32 = derived_fp32_peak(dev, pk) if args.no_probe else fp32_peak(dev, stream)
     fp32_tflops = fp32["fma_f32x2_sustained"]
 
     only = list(range(args.weights)) if args.weights else None
@@ -640,7 +652,8 @@ def run_ours(args, world, rank, local):
     X = torch.from_numpy(X_np).to(dev)
     prod = Product(bsr, weights, X, N, dev)
 
-    res = measure(prod, args.steps, args.warmup, stream, flush, pk, fp32_tflops, hbm, world, local)
+    res = measure(prod, args.steps, args.warmup, stream, flush, pk, fp32_tflops, hbm, world, local,
+                  args.min_seconds)
     K = res["K"]
     total_ms = max_over_ranks(res["total_ms"], world)
     value = world * res["flops"] * K / (total_ms * 1e-3) / 1e9
@@ -687,7 +700,7 @@ def run_ours(args, world, rank, local):
                 ws, Ne = wl.weights, wl.N
                 Xe = dev_array(wl.make_X(), dev)
             pe = Product(bsr, ws, Xe, Ne, dev)
-            r = measure(pe, args.steps, args.warmup, stream, flush, pk, fp32_tflops, hbm, 1, None)
+            r = measure(pe, args.steps, args.warmup, stream, flush, pk, fp32_tflops, hbm, 1, None, args.min_seconds)
             extra[key] = workload_entry(r, pe, hbm, fp32_tflops)
             pe.destroy()
             del Xe
@@ -748,7 +761,7 @@ def run_report(args):
     hbm = float(pk["hbm_gbs"]) * 1e9
     stream = torch.cuda.current_stream()
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
-    fp32 = fp32_peak(dev, stream, sustained_s=0.5)
+    fp32 = derived_fp32_peak(dev, pk) if args.no_probe else fp32_peak(dev, stream, sustained_s=0.5)
     fp32_tflops = fp32["fma_f32x2_sustained"]
     for dt, shape in REPORT_VARIANTS[args.workload]:
         if args.dtype and dt is not None and dt != args.dtype:
@@ -761,7 +774,7 @@ def run_report(args):
             wl.weights = [w for w in wl.weights if f"{w.R}x{w.C}" in args.shapes.split(",")]
         X = dev_array(wl.make_X(), dev)
         prod = Product(bsr, wl.weights, X, wl.N, dev)
-        res = measure(prod, args.steps, args.warmup, stream, flush, pk, fp32_tflops, hbm, 1, 0)
+        res = measure(prod, args.steps, args.warmup, stream, flush, pk, fp32_tflops, hbm, 1, 0, args.min_seconds)
         line = {"workload": args.workload, "name": wl.name}
         line.update(workload_entry(res, prod, hbm, fp32_tflops))
         line["clocks"] = res["clocks"]

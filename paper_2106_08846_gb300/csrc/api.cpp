@@ -121,6 +121,8 @@ Schedule::~Schedule() {
     cudaFree(d_xs_perm);
     cudaFree(d_vmap);
     cudaFree(d_xs_vdst);
+    cudaFree(xr.d_vdst);
+    cudaFree(xr.d_perm);
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);
         cudaFree(tc.d_rec_off[gi]);
@@ -668,12 +670,13 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
              "item_groups=%d\nitems=%zu\nsplit_len=%d\nsplit_rows=%" PRId64 "\nslots=%d\n"
              "empty_rows=%" PRId64 "\nmax_row_blocks=%" PRId64 "\nlaunches_per_call=%d\n"
              "structure_hash=%016" PRIx64 "\ncache_hit=%d\nschedule_reuses=%" PRId64
-             "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\ntc_stacked_chunks=%s\n",
+             "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\ntc_stacked_chunks=%s\n"
+             "xrow_tasks=%d,%d\n",
              variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_R, sc.ex_C, sc.M, sc.K,
              sc.MB, sc.KB, sc.nnzb, sc.tn, sc.threads, sc.smem, sc.groups, sc.items.size(),
              sc.split_len, split_rows, sc.n_slots, sc.empty_rows, sc.max_row, launches_per_call(sc),
              sc.hash, (int)h->cache_hit, (int64_t)sc.reuse_count, (int64_t)g_cache_hits,
-             (int64_t)g_cache_misses, stacks);
+             (int64_t)g_cache_misses, stacks, sc.xr.ok[0] ? sc.xr.n_tasks[0] : 0, sc.xr.ok[1] ? sc.xr.n_tasks[1] : 0);
     return BSR_OK;
 }
 

@@ -12,6 +12,7 @@
 
 #include "bsr.h"
 #include "tc.h"
+#include "xrow.h"
 #include "xstage.h"
 
 namespace bsr {
@@ -61,6 +62,7 @@ struct Schedule {
     std::vector<int32_t> group_begin;   // groups + 1 offsets into items
     XsPlan xs;                          // xstage task footprints
     TcPlan tc;                          // tcgen05 task footprints
+    XrPlan xr;                          // persistent tall-block SIMT kernel (large N), alongside xstage
     int n_slots = 0;
     int64_t empty_rows = 0, max_row = 0;
     int sm_count = 148;
@@ -158,6 +160,11 @@ cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t n
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
                              const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);
+// The persistent tall-block kernel in configuration s (xrow.h).
+cudaError_t launch_xrow(const LaunchArgs &a, int s);
+cudaError_t pack_xrow_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
+                           const int64_t *vdst, int64_t n_items, int64_t nnzb, int R, int C, float *blobs,
+                           cudaStream_t st);
 int launches_per_call(const Schedule &sc);
 
 }  // namespace bsr

@@ -88,7 +88,7 @@ def test_noalloc_capacity_counts_the_executed_block_height():
     w = synth.make_weight("na_rb", 5300, M, K, R, C, "bf16", 0, mask=synth.mask_from_row_counts(5300, cnt, KB))
     h = bsr.bsr_create(*build_on_gpu(w.W, R, C), R, C, M, K)
     sc = h.schedule()
-    assert sc["variant"] == "tc" and sc["exec_R"] == 16 and sc["R"] == 1 and sc["slots"] > 0
+    assert sc["variant"] == "tcgen05" and sc["exec_R"] == 16 and sc["R"] == 1 and sc["slots"] > 0
     n_max = (32 << 20) // (sc["slots"] * sc["exec_R"] * 4)
     g = torch.Generator(device="cuda").manual_seed(5301)
     X = torch.randn((n_max + 1, K), generator=g, device="cuda").to(torch.bfloat16)
