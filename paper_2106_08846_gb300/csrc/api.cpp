@@ -121,8 +121,13 @@ Schedule::~Schedule() {
     cudaFree(d_xs_perm);
     cudaFree(d_vmap);
     cudaFree(d_xs_vdst);
-    cudaFree(xr.d_vdst);
-    cudaFree(xr.d_perm);
+    for (int gi = 0; gi < kGkTaskSizes; gi++) {
+        cudaFree(gk.d_rec[gi]);
+        cudaFree(gk.d_rec_off[gi]);
+        cudaFree(gk.d_wsrc[gi]);
+        cudaFree(gk.d_wslot[gi]);
+        cudaFree(gk.d_wbase[gi]);
+    }
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);
         cudaFree(tc.d_rec_off[gi]);
@@ -664,6 +669,13 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
         snprintf(stacks + at, sizeof stacks - at, gi ? ",%" PRId64 : "%" PRId64,
                  sc.variant == V_TC ? sc.tc.stacks[gi] : (int64_t)0);
     }
+    char gks[64] = "";   // task sizes the gathered-K kernel can run
+    for (int gi = 0; gi < kGkTaskSizes; gi++) {
+        if (sc.gk.off[gi] < 0) continue;
+        const size_t at = strlen(gks);
+        snprintf(gks + at, sizeof gks - at, at ? ",%d" : "%d", kGkG[gi]);
+    }
+    if (!gks[0]) snprintf(gks, sizeof gks, "none");
     snprintf(buf, len,
              "variant=%s\ndtype=%s\nR=%d\nC=%d\nexec_R=%d\nexec_C=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
              "\nKB=%" PRId64 "\nnnzb=%" PRId64 "\ntokens_per_cta=%d\nthreads=%d\nsmem_bytes=%zu\n"
@@ -671,12 +683,12 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
              "empty_rows=%" PRId64 "\nmax_row_blocks=%" PRId64 "\nlaunches_per_call=%d\n"
              "structure_hash=%016" PRIx64 "\ncache_hit=%d\nschedule_reuses=%" PRId64
              "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\ntc_stacked_chunks=%s\n"
-             "xrow_tasks=%d,%d\n",
+             "gk_task_sizes=%s\n",
              variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_R, sc.ex_C, sc.M, sc.K,
              sc.MB, sc.KB, sc.nnzb, sc.tn, sc.threads, sc.smem, sc.groups, sc.items.size(),
              sc.split_len, split_rows, sc.n_slots, sc.empty_rows, sc.max_row, launches_per_call(sc),
              sc.hash, (int)h->cache_hit, (int64_t)sc.reuse_count, (int64_t)g_cache_hits,
-             (int64_t)g_cache_misses, stacks, sc.xr.ok[0] ? sc.xr.n_tasks[0] : 0, sc.xr.ok[1] ? sc.xr.n_tasks[1] : 0);
+             (int64_t)g_cache_misses, stacks, gks);
     return BSR_OK;
 }
 

@@ -11,8 +11,8 @@
 #include <vector>
 
 #include "bsr.h"
+#include "gk.h"
 #include "tc.h"
-#include "xrow.h"
 #include "xstage.h"
 
 namespace bsr {
@@ -62,7 +62,7 @@ struct Schedule {
     std::vector<int32_t> group_begin;   // groups + 1 offsets into items
     XsPlan xs;                          // xstage task footprints
     TcPlan tc;                          // tcgen05 task footprints
-    XrPlan xr;                          // persistent tall-block SIMT kernel (large N), alongside xstage
+    GkPlan gk;                          // gathered-K tensor-core kernel, alongside the variant's own
     int n_slots = 0;
     int64_t empty_rows = 0, max_row = 0;
     int sm_count = 148;
@@ -160,12 +160,12 @@ cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t n
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
                              const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);
-// The persistent tall-block kernel in configuration s (xrow.h).
-cudaError_t launch_xrow(const LaunchArgs &a, int s);
-cudaError_t pack_xrow_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
-                           const int64_t *vdst, int64_t n_items, int64_t nnzb, int R, int C, float *blobs,
-                           cudaStream_t st);
-int launches_per_call(const Schedule &sc);
+// The gathered-K tensor-core kernel at task size G (gk.h).
+cudaError_t launch_gk(const LaunchArgs &a, int G);
+cudaError_t pack_gk_data(const void *data, bsr_dtype_t dt, const int32_t *wsrc, const int32_t *wslot,
+                         const int64_t *wbase, int64_t n, int R, int C, void *out, cudaStream_t s);
+
+int launches_per_call(const Schedule &sc, int64_t N = 0);   // N = 0: the schedule variant's own path
 
 }  // namespace bsr
 

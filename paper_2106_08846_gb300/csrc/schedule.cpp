@@ -16,6 +16,7 @@
 #include <queue>
 #include <string>
 
+#include "gk_plan.h"
 #include "schedule.h"
 
 namespace bsr {
@@ -253,120 +254,6 @@ void plan_xstage(Schedule &sc) {
             }
         }
     }
-}
-
-// The persistent tall-block kernel (spmm_xrow.cu), both configurations:
-// tasks of G consecutive items of the (longest-first) item list, so a task's
-// items have similar lengths and its warps finish each chunk together; per
-// item a record (per chunk its first block; per block its X offset in a stage
-// or its block column; one-column blocks ordered inside each chunk so that
-// aligned groups of four have distinct bank residues) and its values; per
-// task the work of one unit, the multiply-adds per token of its longest item
-// plus a fixed cost (the epilogue, about one 32-row block per 16 outputs),
-// as prefix sums. The blobs follow the xstage blobs in the packed values.
-void plan_xrow(Schedule &sc) {
-    XrPlan &pl = sc.xr;
-    for (int s = 0; s < kXrConfigs; s++) {
-        pl.ok[s] = false;
-        pl.n_tasks[s] = 0;
-        pl.blob_off[s] = pl.cost_off[s] = -1;
-    }
-    pl.blob.clear();
-    pl.vdst.clear();
-    pl.perm.clear();
-    pl.total_bytes = 0;
-    const int64_t n = (int64_t)sc.items.size();
-    if (!xrow_supports(sc.R, sc.C, sc.dt, sc.K) || n == 0 || sc.nnzb == 0) return;
-    const int64_t per_block = xrow_block_floats(sc.R, sc.C);
-    const int64_t base = ((int64_t)sc.xs_blob.size() * 4 + 255) & ~int64_t(255);   // bytes into the packed values
-    pl.vdst.assign((size_t)(kXrConfigs * n), -1);
-    pl.perm.assign((size_t)(kXrConfigs * sc.nnzb), 0);
-    std::vector<int32_t> words;   // the region after base, as int32
-    for (int s = 0; s < kXrConfigs; s++) {
-        const int G = xrow_G(s), KC = xrow_chunk(s), TN = xrow_tokens(s);
-        const int64_t nch = (sc.K + KC - 1) / KC;
-        int32_t *perm = pl.perm.data() + (size_t)s * sc.nnzb;
-        std::vector<std::vector<int32_t>> recs((size_t)n);
-        for (int64_t i = 0; i < n; i++) {
-            const Item &it = sc.items[(size_t)i];
-            const int32_t len = it.p1 - it.p0;
-            std::vector<int32_t> &r = recs[(size_t)i];
-            r.assign((size_t)(xstage_pad4(nch + 1) + xstage_pad4(len)), 0);
-            for (int32_t k = 0; k < len; k++) perm[it.p0 + k] = it.p0 + k;
-            int32_t b = 0;
-            for (int64_t c = 0; c <= nch; c++) {
-                while (b < len && (int64_t)sc.indices[it.p0 + b] * sc.C < c * KC) b++;
-                r[(size_t)c] = b;
-            }
-            if (sc.C == 1)
-                for (int64_t c = 0; c < nch; c++) quad_order(sc, perm + it.p0, r[(size_t)c], r[(size_t)c + 1]);
-            const size_t at = (size_t)xstage_pad4(nch + 1);
-            for (int32_t k = 0; k < len; k++) {
-                const int64_t col = sc.indices[perm[it.p0 + k]];
-                r[at + (size_t)k] = sc.C == 1 ? (int32_t)xrow_stage_offset(sc.dt, TN, (int)(col % KC)) : (int32_t)col;
-            }
-        }
-        const int64_t n_tasks = (n + G - 1) / G;
-        size_t ib = 0, wb = 0;
-        for (int64_t t = 0; t < n_tasks; t++) {
-            size_t ri = 0, wi = 0;
-            for (int64_t i = t * G; i < std::min(n, (t + 1) * G); i++) {
-                ri += recs[(size_t)i].size() * 4;
-                wi += (size_t)(sc.items[(size_t)i].p1 - sc.items[(size_t)i].p0) * per_block * 4;
-            }
-            ib = std::max(ib, ri);
-            wb = std::max(wb, wi);
-        }
-        ib = (ib + 15) & ~size_t(15);
-        wb = (wb + 15) & ~size_t(15);
-        const size_t hdr = (size_t)G * kXrItab * 4;
-        const size_t stride = hdr + ib + wb;
-        if (xrow_smem_bytes(s, sc.dt, stride) > (size_t)kXrMaxSmem || stride > UINT32_MAX) continue;
-        // blobs
-        const size_t blob_at = (words.size() * 4 + 255) & ~size_t(255);
-        words.resize((blob_at + (size_t)n_tasks * stride) / 4, 0);
-        std::vector<int64_t> cost((size_t)n_tasks + 1, 0);
-        for (int64_t t = 0; t < n_tasks; t++) {
-            const size_t b0 = blob_at + (size_t)t * stride;
-            int64_t roff = 0, woff = 0, longest = 0;
-            for (int64_t k = 0; k < G && t * G + k < n; k++) {
-                const int64_t i = t * G + k;
-                const Item &it = sc.items[(size_t)i];
-                const int64_t len = it.p1 - it.p0;
-                int32_t *h = &words[(b0 + (size_t)k * kXrItab * 4) / 4];
-                h[0] = it.row;
-                h[1] = it.slot;
-                h[2] = (int32_t)len;
-                h[3] = (int32_t)woff;
-                h[4] = (int32_t)roff;
-                const std::vector<int32_t> &r = recs[(size_t)i];
-                std::copy(r.begin(), r.end(), words.begin() + (ptrdiff_t)((b0 + hdr) / 4 + (size_t)roff));
-                if (len) pl.vdst[(size_t)(s * n + i)] = (base + (int64_t)(b0 + hdr + ib)) / 4 + woff;
-                roff += (int64_t)r.size();
-                woff += len * per_block;
-                longest = std::max(longest, len);
-            }
-            cost[(size_t)t + 1] = cost[(size_t)t] + longest * sc.R * sc.C + 32 * sc.R;
-        }
-        // the prefix sums of the per-unit work
-        const size_t cost_at = (words.size() * 4 + 255) & ~size_t(255);
-        words.resize((cost_at + cost.size() * 8) / 4, 0);
-        std::copy(cost.begin(), cost.end(), reinterpret_cast<int64_t *>(words.data() + cost_at / 4));
-        pl.ok[s] = true;
-        pl.n_tasks[s] = (int)n_tasks;
-        pl.stride[s] = (uint32_t)stride;
-        pl.ibytes[s] = (uint32_t)ib;
-        pl.wbytes[s] = (uint32_t)wb;
-        pl.blob_off[s] = base + (int64_t)blob_at;
-        pl.cost_off[s] = base + (int64_t)cost_at;
-    }
-    if (!pl.ok[0] && !pl.ok[1]) {
-        pl.vdst.clear();
-        pl.perm.clear();
-        return;
-    }
-    pl.blob.swap(words);
-    pl.total_bytes = base + (int64_t)pl.blob.size() * 4;
 }
 
 // Tasks of the tensor-core kernel for every task size G: ceil(items / G)
@@ -618,9 +505,16 @@ bsr_status_t build_schedule(Schedule &sc) {
         limit = limit ? std::min(limit, lmax) : (sc.max_row > lmax ? lmax : 0);
         make_items(sc, limit, sc.R > 1);   // one-row blocks keep their rare empty rows: tasks stay row-contiguous
         plan_xstage(sc);
-        plan_xrow(sc);
     }
     if (sc.variant == V_XSTAGE && (int64_t)sc.xs_blob.size() > INT32_MAX) sc.variant = V_GENERIC;   // blob offsets are int32
+    // the gathered-K kernel, after the variant's own packed values (the
+    // generic kernel's: a copy of the caller's block values)
+    if (sc.variant == V_TC)
+        plan_gk(sc, sc.tc_w_total);
+    else if (sc.variant == V_XSTAGE)
+        plan_gk(sc, (int64_t)sc.xs_blob.size() * 4);
+    else
+        plan_gk(sc, sc.nnzb * sc.R * sc.C * (int64_t)dtype_size(sc.dt));
     if (sc.variant == V_GENERIC) {
         sc.threads = 256;
         sc.xs_rec.clear();
@@ -636,11 +530,19 @@ bsr_status_t build_schedule(Schedule &sc) {
         upload(&sc.d_group_begin, sc.group_begin) != cudaSuccess ||
         upload(&sc.d_indptr, sc.indptr) != cudaSuccess || upload(&sc.d_indices, sc.indices) != cudaSuccess ||
         upload(&sc.d_xs_perm, sc.xs_perm) != cudaSuccess || upload(&sc.d_xs_vdst, sc.xs_vdst) != cudaSuccess ||
-        upload(&sc.d_vmap, sc.vmap) != cudaSuccess || upload(&sc.xr.d_vdst, sc.xr.vdst) != cudaSuccess ||
-        upload(&sc.xr.d_perm, sc.xr.perm) != cudaSuccess) {
+        upload(&sc.d_vmap, sc.vmap) != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_ALLOC;
     }
+    for (int gi = 0; gi < kGkTaskSizes; gi++)
+        if (upload(&sc.gk.d_rec[gi], sc.gk.rec[gi]) != cudaSuccess ||
+            upload(&sc.gk.d_rec_off[gi], sc.gk.rec_off[gi]) != cudaSuccess ||
+            upload(&sc.gk.d_wsrc[gi], sc.gk.wsrc[gi]) != cudaSuccess ||
+            upload(&sc.gk.d_wslot[gi], sc.gk.wslot[gi]) != cudaSuccess ||
+            upload(&sc.gk.d_wbase[gi], sc.gk.wbase[gi]) != cudaSuccess) {
+            cudaGetLastError();
+            return BSR_ERR_ALLOC;
+        }
     for (int gi = 0; gi < kTcTaskSizes; gi++)
         if (upload(&sc.tc.d_rec[gi], sc.tc.rec[gi]) != cudaSuccess ||
             upload(&sc.tc.d_rec_off[gi], sc.tc.rec_off[gi]) != cudaSuccess ||
@@ -655,12 +557,13 @@ bsr_status_t build_schedule(Schedule &sc) {
 bsr_status_t pack_data(Handle &h) {
     h.data_packed = nullptr;
     const Schedule &sc = *h.sched;
-    if (sc.variant == V_TC && sc.ex_nnzb == 0) return BSR_OK;
-    if (sc.variant != V_XSTAGE && sc.variant != V_TC) return BSR_OK;
+    if (sc.variant == V_TC && sc.ex_nnzb == 0 && !sc.gk.ok) return BSR_OK;
+    if (sc.variant != V_XSTAGE && sc.variant != V_TC && !sc.gk.ok) return BSR_OK;
+    const size_t raw_bytes = (size_t)sc.nnzb * sc.R * sc.C * dtype_size(sc.dt);
     // xstage: the task blobs (item tables and records from the schedule's
     // template, then this handle's block values)
-    const size_t bytes = sc.variant == V_TC ? (size_t)sc.tc_w_total
-                                            : std::max(sc.xs_blob.size() * 4, (size_t)sc.xr.total_bytes);
+    size_t bytes = sc.variant == V_TC ? (size_t)sc.tc_w_total : sc.variant == V_XSTAGE ? sc.xs_blob.size() * 4 : raw_bytes;
+    if (sc.gk.ok) bytes = std::max(bytes, (size_t)sc.gk.total_bytes);
     if (bytes == 0) return BSR_OK;
     if (cudaMalloc(&h.data_packed, bytes) != cudaSuccess) {
         cudaGetLastError();
@@ -694,18 +597,25 @@ bsr_status_t pack_data(Handle &h) {
                                      (int64_t)sc.tc.worder[gi].size(), sc.R, sc.C,
                                      (unsigned char *)h.data_packed + sc.tc.w_off[gi], 0);
         }
+    } else if (sc.variant != V_XSTAGE) {
+        // the generic kernel reads the block values from the start of the packed buffer
+        e = cudaMemcpy(h.data_packed, h.data, raw_bytes, cudaMemcpyDeviceToDevice);
     } else {
         e = cudaMemcpy(h.data_packed, sc.xs_blob.data(), sc.xs_blob.size() * 4, cudaMemcpyHostToDevice);
-        if (e == cudaSuccess && !sc.xr.blob.empty())
-            e = cudaMemcpy((unsigned char *)h.data_packed + (sc.xr.total_bytes - (int64_t)sc.xr.blob.size() * 4),
-                           sc.xr.blob.data(), sc.xr.blob.size() * 4, cudaMemcpyHostToDevice);
         if (e == cudaSuccess && sc.nnzb > 0)
             e = pack_xstage_data(h.data, sc.dt, sc.d_items, sc.d_xs_perm, sc.d_xs_vdst, (int64_t)sc.items.size(),
                                  sc.R, sc.C, (float *)h.data_packed, 0);
-        if (e == cudaSuccess && sc.nnzb > 0 && !sc.xr.blob.empty())
-            e = pack_xrow_data(h.data, sc.dt, sc.d_items, sc.xr.d_perm, sc.xr.d_vdst, (int64_t)sc.items.size(),
-                               sc.nnzb, sc.R, sc.C, (float *)h.data_packed, 0);
     }
+    // the gathered-K kernel's operands: zero padding, then the block values
+    int64_t gk_lo = -1;
+    for (int gi = 0; gi < kGkTaskSizes; gi++)
+        if (sc.gk.off[gi] >= 0 && (gk_lo < 0 || sc.gk.off[gi] < gk_lo)) gk_lo = sc.gk.off[gi];
+    if (e == cudaSuccess && gk_lo >= 0)
+        e = cudaMemset((unsigned char *)h.data_packed + gk_lo, 0, (size_t)(sc.gk.total_bytes - gk_lo));
+    for (int gi = 0; gi < kGkTaskSizes && e == cudaSuccess; gi++)
+        if (sc.gk.off[gi] >= 0)
+            e = pack_gk_data(h.data, sc.dt, sc.gk.d_wsrc[gi], sc.gk.d_wslot[gi], sc.gk.d_wbase[gi],
+                             (int64_t)sc.gk.wsrc[gi].size(), sc.R, sc.C, h.data_packed, 0);
     if (e != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
         cudaGetLastError();
         return BSR_ERR_CUDA;
@@ -713,7 +623,10 @@ bsr_status_t pack_data(Handle &h) {
     return BSR_OK;
 }
 
-int launches_per_call(const Schedule &sc) { return 1 + (sc.splits.empty() ? 0 : 1); }
+int launches_per_call(const Schedule &sc, int64_t N) {
+    if (choose_gk(sc, N) >= 0) return 1;   // no split rows, no reduce pass
+    return 1 + (sc.splits.empty() ? 0 : 1);
+}
 
 // Task size for this call: the G that minimises a simple cost model,
 // waves * (fixed CTA cost + the work of G items), among the G whose shared
@@ -785,27 +698,8 @@ int choose_tc_tasks(const Schedule &sc, int64_t N) {
     return best;
 }
 
-// The persistent tall-block kernel's configuration for this call, or -1
-// for the xstage kernel: it runs when every SM gets at least one unit (a
-// task on one token tile), the 64-token configuration first (its stages
-// hold 128 columns: fewer chunk boundaries per unit). BSR_XROW=0 in the
-// environment turns it off, BSR_XROW=1 uses it whenever a configuration fits.
-int choose_xrow(const Schedule &sc, int64_t N) {
-    static const int mode = [] {
-        const char *v = getenv("BSR_XROW");
-        return v ? atoi(v) : -1;
-    }();
-    if (mode == 0 || sc.variant != V_XSTAGE) return -1;
-    for (int s = 0; s < kXrConfigs; s++) {
-        if (!sc.xr.ok[s]) continue;
-        const int64_t units = (int64_t)sc.xr.n_tasks[s] * ((N + xrow_tokens(s) - 1) / xrow_tokens(s));
-        if (mode == 1 || units >= sc.sm_count) return s;
-    }
-    return -1;
-}
-
 int fusion_class(const Schedule &sc, int64_t N, int *G) {
-    if (sc.variant == V_XSTAGE && choose_xrow(sc, N) >= 0) {   // a persistent grid of its own
+    if (choose_gk(sc, N) >= 0) {   // a grid of its own
         *G = 0;
         return -1;
     }
@@ -860,13 +754,13 @@ cudaError_t launch_spmm_batch(const LaunchArgs *as, int n) {
 }
 
 cudaError_t launch_spmm(const LaunchArgs &a) {
+    const int gG = choose_gk(*a.sc, a.N);
+    if (gG >= 0) return launch_gk(a, gG);   // every block row is an item: nothing to reduce
     cudaError_t e;
     if (a.sc->variant == V_TC)
         e = launch_tc(a, choose_tc_tasks(*a.sc, a.N));
-    else if (a.sc->variant == V_XSTAGE) {
-        const int s = choose_xrow(*a.sc, a.N);
-        e = s >= 0 ? launch_xrow(a, s) : launch_xstage(a, choose_tasks(*a.sc, a.N));
-    }
+    else if (a.sc->variant == V_XSTAGE)
+        e = launch_xstage(a, choose_tasks(*a.sc, a.N));
     else
         e = launch_generic(a);
     if (e != cudaSuccess) return e;

@@ -13,10 +13,6 @@ bsr_status_t build_schedule(Schedule &sc);
 // kernel wants one (else the borrowed array is used directly).
 bsr_status_t pack_data(Handle &h);
 
-// The persistent tall-block kernel's configuration for a call of N tokens,
-// or -1 when the xstage kernel runs it.
-int choose_xrow(const Schedule &sc, int64_t N);
-
 // Launches every kernel of one bsr_spmm call on a.stream.
 cudaError_t launch_spmm(const LaunchArgs &a);
 
