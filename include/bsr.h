@@ -20,7 +20,8 @@
  * and Y, fp32 accumulation) or BSR_BF16 (bf16 data, X and Y, fp32
  * accumulation, Y rounded to nearest even). bias is always fp32 or NULL.
  * Plain TF32 is never used for BSR_F32. fp32 blocks of 32 or more rows with
- * 16 or 32 columns run on the tensor cores as 3xTF32: each operand is split
+ * 16 or 32 columns, and 16-row blocks of such width in weights of at least
+ * 2^20 elements (M K), run on the tensor cores as 3xTF32: each operand is split
  * into a tf32 high part and a tf32 low part (the remainder) and the product is
  * hi*hi + hi*lo + lo*hi, accumulated in fp32. The dropped lo*lo term and the
  * rounding of the low parts leave a relative error near 2^-20 per product,

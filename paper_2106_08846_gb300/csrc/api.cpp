@@ -133,6 +133,8 @@ Schedule::~Schedule() {
         cudaFree(tc.d_rec_off[gi]);
         cudaFree(tc.d_worder[gi]);
         cudaFree(tc.d_wstack[gi]);
+        cudaFree(tc.d_prog[gi]);
+        cudaFree(tc.d_stab[gi]);
     }
     cudaFree(d_indices);
 }

@@ -160,6 +160,10 @@ cudaError_t reblock_tc_data(const uint16_t *data, const int32_t *vmap, int64_t n
 cudaError_t pack_xstage_data(const void *data, bsr_dtype_t dt, const Item *items, const int32_t *perm,
                              const int64_t *vdst, int64_t n_items, int R, int C, float *blobs, cudaStream_t s);
 cudaError_t launch_reduce(const LaunchArgs &a);
+// The persistent tensor-core kernel on the tc task records at task size G,
+// and the task size it runs a call of N tokens at (-1: the tc kernel runs it).
+cudaError_t launch_tcp(const LaunchArgs &a, int G);
+int choose_tcp(const Schedule &sc, int64_t N);
 // The gathered-K tensor-core kernel at task size G (gk.h).
 cudaError_t launch_gk(const LaunchArgs &a, int G);
 cudaError_t pack_gk_data(const void *data, bsr_dtype_t dt, const int32_t *wsrc, const int32_t *wslot,

@@ -186,7 +186,7 @@ void footprints(const Schedule &sc, size_t per_block, int chunk, const int *Gs, 
     const int64_t nch = (sc.K + chunk - 1) / chunk;
     for (int gi = 0; gi < nG; gi++) {
         const int G = Gs[gi];
-        size_t wmax = 0, imax = 0;
+        size_t wmax = 0, imax = 0, swmax = 0;
         for (size_t t = 0; t < sc.items.size(); t += G) {
             size_t blocks = 0, rec = 0;
             for (size_t k = t; k < std::min(sc.items.size(), t + G); k++) {
@@ -287,7 +287,7 @@ void plan_tc(Schedule &sc) {
         stack.clear();
         sc.tc.task_cost_max[gi] = 0;
         sc.tc.stacks[gi] = 0;
-        size_t wmax = 0, imax = 0;
+        size_t wmax = 0, imax = 0, swmax = 0;
         const int64_t n_tasks = (n_items + G - 1) / G;
         std::vector<std::vector<int32_t>> members((size_t)n_tasks);
         {
@@ -331,6 +331,12 @@ void plan_tc(Schedule &sc) {
                 wmax = std::max(wmax, per_chunk[(size_t)c].size() * per_block);
             }
             rec[head + 4 + (size_t)nch] = n;
+            for (int64_t c0 = 0; c0 < nch; c0 += tcp_stage_chunks(sc.dt)) {
+                size_t nb = 0;
+                for (int64_t c = c0; c < std::min<int64_t>(nch, c0 + tcp_stage_chunks(sc.dt)); c++)
+                    nb += per_chunk[(size_t)c].size();
+                swmax = std::max(swmax, nb * per_block);
+            }
             // stacks, and the task's MMA cost
             double cost = 0.0;
             for (int64_t c = 0; c < nch; c++) {
@@ -365,6 +371,7 @@ void plan_tc(Schedule &sc) {
             imax = std::max(imax, (rec.size() - head) * 4);
         }
         sc.tc.task_wbytes[gi] = (wmax + 15) & ~size_t(15);
+        sc.tc.tcp_wbytes[gi] = (swmax + 15) & ~size_t(15);
         sc.tc.task_ibytes[gi] = imax;
         const bool ok = G * sc.R <= kTcTmemCols &&
                         tc_smem_bytes(sc.R, G, sc.tc.task_wbytes[gi], imax, sc.dt) <= (size_t)kTcMaxSmem &&
@@ -453,10 +460,10 @@ bsr_status_t build_schedule(Schedule &sc) {
     sc.ex_nnzb = sc.nnzb;
     std::vector<int32_t> tptr, tind;
     int RT = sc.R;
-    const bool reblock = !want_generic && !want_xstage && !tc_supports(sc.R, sc.C, sc.dt, sc.K) &&
+    const bool reblock = !want_generic && !want_xstage && !tc_supports(sc.R, sc.C, sc.dt, sc.K, sc.M * sc.K) &&
                          reblock_for_tc(sc, tptr, tind, sc.vmap, &RT);
     if (!reblock) sc.vmap.clear();
-    if (!want_generic && !want_xstage && (reblock || tc_supports(sc.R, sc.C, sc.dt, sc.K))) {
+    if (!want_generic && !want_xstage && (reblock || tc_supports(sc.R, sc.C, sc.dt, sc.K, sc.M * sc.K))) {
         // plan on the tile structure (the user's arrays stay the cache key)
         std::vector<int32_t> uptr, uind;
         const int uC = sc.C, uR = sc.R;
@@ -478,10 +485,11 @@ bsr_status_t build_schedule(Schedule &sc) {
         }
         sc.variant = V_TC;
         sc.tn = kTcTokens;
-        sc.threads = 192;
+        sc.threads = tc_threads(sc.dt == BSR_F32);
         // block values stream per chunk: only balance decides the splitting
         make_items(sc, split_limit(sc), true);
         plan_tc(sc);
+        plan_tcp(sc);
         if (reblock) {
             sc.indptr.swap(uptr);
             sc.indices.swap(uind);
@@ -547,7 +555,9 @@ bsr_status_t build_schedule(Schedule &sc) {
         if (upload(&sc.tc.d_rec[gi], sc.tc.rec[gi]) != cudaSuccess ||
             upload(&sc.tc.d_rec_off[gi], sc.tc.rec_off[gi]) != cudaSuccess ||
             upload(&sc.tc.d_worder[gi], sc.tc.worder[gi]) != cudaSuccess ||
-            upload(&sc.tc.d_wstack[gi], sc.tc.wstack[gi]) != cudaSuccess) {
+            upload(&sc.tc.d_wstack[gi], sc.tc.wstack[gi]) != cudaSuccess ||
+            upload(&sc.tc.d_prog[gi], sc.tc.prog[gi]) != cudaSuccess ||
+            upload(&sc.tc.d_stab[gi], sc.tc.stab[gi]) != cudaSuccess) {
             cudaGetLastError();
             return BSR_ERR_ALLOC;
         }
@@ -708,6 +718,10 @@ int fusion_class(const Schedule &sc, int64_t N, int *G) {
         return 2 * xstage_fusion_key(sc, *G);
     }
     if (sc.variant == V_TC) {
+        if (choose_tcp(sc, N) >= 0) {   // persistent: a grid of its own
+            *G = 0;
+            return -1;
+        }
         *G = choose_tc_tasks(sc, N);
         return 2 * tc_fusion_key(sc) + 1;
     }
@@ -757,7 +771,10 @@ cudaError_t launch_spmm(const LaunchArgs &a) {
     const int gG = choose_gk(*a.sc, a.N);
     if (gG >= 0) return launch_gk(a, gG);   // every block row is an item: nothing to reduce
     cudaError_t e;
-    if (a.sc->variant == V_TC)
+    const int tG = a.sc->variant == V_TC ? choose_tcp(*a.sc, a.N) : -1;
+    if (tG >= 0)
+        e = launch_tcp(a, tG);
+    else if (a.sc->variant == V_TC)
         e = launch_tc(a, choose_tc_tasks(*a.sc, a.N));
     else if (a.sc->variant == V_XSTAGE)
         e = launch_xstage(a, choose_tasks(*a.sc, a.N));

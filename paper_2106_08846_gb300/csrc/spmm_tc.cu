@@ -42,6 +42,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <cstdlib>
 #include <mutex>
 
 #include "bsr_internal.h"
@@ -62,9 +63,9 @@ template <typename T>
 struct TcCfg {
     static constexpr int KC = 128 / (int)sizeof(T);
     static constexpr int NS = sizeof(T) == 4 ? kTcStagesF32 : kTcStages;
+    static constexpr int NISS = tc_issuers(sizeof(T) == 4);   // MMA-issuing warps (lane 0 of each)
+    static constexpr int NTHREADS = tc_threads(sizeof(T) == 4);
 };
-constexpr int NWARPS = 6;
-constexpr int NTHREADS = NWARPS * 32;
 constexpr uint64_t kDrainNs = 200000000ull;
 
 struct TcArgs {
@@ -161,6 +162,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
     ptx::pdl_launch_dependents();
     constexpr bool F32 = sizeof(T) == 4;
     constexpr int NS = TcCfg<T>::NS;
+    constexpr int NISS = TcCfg<T>::NISS;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *base =
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -187,10 +189,10 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; s++) {
             ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], 1);
+            ptx::mbar_init(&empty[s], NISS);
             ptx::mbar_init(&split[s], 1);
         }
-        ptx::mbar_init(done, 1);
+        ptx::mbar_init(done, NISS);
         ptx::mbar_init(rbar, 1);
         misc[0] = 0;
         ptx::fence_barrier_init();
@@ -260,9 +262,32 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                 if (d != stalled) ptx::mbar_wait_bounded(&full[d % NS], (d / NS) & 1, kDrainNs);
             ptx::mbar_wait_bounded(rbar, 0, kDrainNs);
         }
-    } else if (warp == 1) {
-        // ---------------- MMA issuer
+    } else if (warp <= NISS) {
+        // ---------------- MMA issuers: lane 0 of warps 1..NISS, each over a
+        // contiguous range of the task's items (its accumulators), ranges
+        // balanced by block count; every issuer walks every chunk and
+        // commits the stage, so `empty` and `done` count NISS arrivals
         if (lane == 0) {
+            const int q = warp - 1;
+            int i0 = 0, i1 = 0;
+            {
+                int total = 0;
+                for (int g = 0; g < g_count; g++) total += itab[6 * g + 5];
+                int acc = 0;
+                i0 = g_count;
+                for (int g = 0; g < g_count; g++) {
+                    const int len = itab[6 * g + 5];
+                    const int owner =
+                        total > 0 ? min(NISS - 1, (int)((int64_t)(2 * acc + len) * NISS / (2 * (int64_t)total))) : 0;
+                    acc += len;
+                    if (owner == q) {
+                        i0 = min(i0, g);
+                        i1 = g + 1;
+                    }
+                }
+                if (i1 == 0) i0 = 0;
+            }
+            const uint32_t ufirst = (uint32_t)i0, ucnt = (uint32_t)(i1 - i0);
             bool ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns) && !aborted(misc);
             const int32_t *ent = I_s + items_at + 4 * g_count;
             int k = 0;   // chunks consumed
@@ -284,11 +309,12 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                 const uint64_t a0 = umma_desc(stage, 16, 1024, 2), b0 = umma_desc(w_stage, 128, 256, 0);
                 const uint32_t wb16 = wblock >> 4;
                 int e = lo;
-                if constexpr (!F32) {
+                if constexpr (!F32 && NISS == 1) {
                     if (C == 16) {
-                        // one MMA per block: read and decode 4 entries, then
-                        // issue their MMAs back to back (one thread issues,
-                        // so the decoding would otherwise sit between MMAs)
+                        // one issuer, one MMA per block: read and decode 4
+                        // entries, then issue their MMAs back to back (one
+                        // thread issues, so the decoding would otherwise sit
+                        // between MMAs)
                         constexpr uint32_t idesc = idesc_bf16(TN, R);
                         for (; e + 4 <= hi; e += 4) {
                             const uint32_t vv[4] = {(uint32_t)ent[e], (uint32_t)ent[e + 1], (uint32_t)ent[e + 2],
@@ -296,22 +322,39 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                             uint64_t adv[4], bdv[4];
                             uint32_t dv[4], acc[4];
 #pragma unroll
-                            for (int j = 0; j < 4; j++) {
-                                adv[j] = a0 + (uint64_t)((vv[j] & 3u) * 2u);
-                                bdv[j] = b0 + (uint64_t)((uint32_t)(e + j - lo) * wb16);
-                                dv[j] = tmem + ((vv[j] >> 2) & 31u) * R;
-                                acc[j] = ((vv[j] >> 7) & 1u) == 0u;
+                            for (int jj = 0; jj < 4; jj++) {
+                                adv[jj] = a0 + (uint64_t)((vv[jj] & 3u) * 2u);
+                                bdv[jj] = b0 + (uint64_t)((uint32_t)(e + jj - lo) * wb16);
+                                dv[jj] = tmem + ((vv[jj] >> 2) & 31u) * R;
+                                acc[jj] = ((vv[jj] >> 7) & 1u) == 0u;
                             }
 #pragma unroll
-                            for (int j = 0; j < 4; j++) mma_bf16(dv[j], adv[j], bdv[j], idesc, acc[j]);
+                            for (int jj = 0; jj < 4; jj++) mma_bf16(dv[jj], adv[jj], bdv[jj], idesc, acc[jj]);
                         }
                     }
                 }
-                for (; e < hi; e++) {
+                for (; ucnt > 0 && e < hi; e++) {
                     const uint32_t v = (uint32_t)ent[e];
                     const uint32_t g = (v >> 2) & 31u, first = (v >> 7) & 1u;
                     const uint64_t ad = a0 + (uint64_t)((v & 3u) * 2u);             // + (v & 3) * 32 bytes
                     const uint64_t bd = b0 + (uint64_t)((uint32_t)(e - lo) * wb16);
+                    if constexpr (!F32) {
+                        if ((v >> 9) & 1u) continue;   // a stack member: its rows are in its head's MMAs
+                        if ((v >> 8) & 1u) {
+                            // a stack head: the B operand of all g_count items'
+                            // blocks; this issuer's items are rows ufirst*R ..
+                            // of it, into their adjacent accumulators
+                            const uint32_t ns = (uint32_t)(g_count * R);
+                            const uint32_t idesc_s = idesc_bf16(TN, (int)(ucnt * R));
+                            const uint64_t bs = bd + (uint64_t)(ufirst * R * 2);   // ufirst * R rows of 32 bytes
+#pragma unroll 4
+                            for (int sl = 0; sl < C / 16; sl++)
+                                mma_bf16(tmem + ufirst * R, ad + (uint64_t)(sl * 2), bs + (uint64_t)(sl * ns * 2),
+                                         idesc_s, (first == 0u) | (sl > 0));
+                            continue;
+                        }
+                    }
+                    if (g - ufirst >= ucnt) continue;   // another issuer's item
                     const uint32_t d = tmem + g * R;
                     if constexpr (F32) {
                         // 3xTF32: high x high + high x low + low x high, K = 8 per MMA
@@ -326,40 +369,25 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                         }
                     } else {
                         constexpr uint32_t idesc = idesc_bf16(TN, R);
-                        if (C == 16) {   // (one MMA per block: handled in batches below)
-                            mma_bf16(d, ad, bd, idesc, first == 0u);
-                        } else if ((v >> 9) & 1u) {
-                            // a stack member: its rows are in its head's MMAs
-                        } else if ((v >> 8) & 1u) {
-                            // a stack head: the B operand of all g_count items' blocks,
-                            // into their adjacent accumulators
-                            const uint32_t ns = (uint32_t)(g_count * R);
-                            const uint32_t idesc_s = idesc_bf16(TN, (int)ns);
 #pragma unroll 4
-                            for (int sl = 0; sl < C / 16; sl++)
-                                mma_bf16(tmem, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * ns * 2), idesc_s,
-                                         (first == 0u) | (sl > 0));
-                        } else {
-#pragma unroll 4
-                            for (int sl = 0; sl < C / 16; sl++)
-                                mma_bf16(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
-                                         (first == 0u) | (sl > 0));
-                        }
+                        for (int sl = 0; sl < C / 16; sl++)
+                            mma_bf16(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
+                                     (first == 0u) | (sl > 0));
                     }
                 }
-                mma_commit(&empty[s]);   // the stage is free once these MMAs completed
+                mma_commit(&empty[s]);   // the stage is free once every issuer's MMAs completed
                 k++;
             }
             if (!ok) {
                 set_status(a.status, DEV_TIMEOUT);
                 atomicExch(&misc[0], 1);
             }
-            mma_commit(done);   // every MMA issued above completes before `done`
+            mma_commit(done);   // every MMA this issuer issued completes before its `done` arrival
         }
     } else {
-        // ---------------- warps 2..5: fp32 split during the main loop, then
-        // the epilogue; TMEM lane quarter = warp % 4
-        const int et = threadIdx.x - 64;   // 0..127
+        // ---------------- the last four warps: fp32 split during the main
+        // loop, then the epilogue; TMEM lane quarter = warp % 4
+        const int et = threadIdx.x - 32 * (1 + NISS);   // 0..127
         ptx::pdl_wait();   // the bias, Y and the workspace may be an earlier kernel's
         for (int e = et; e < g_count * R; e += 128) {
             const int g = e / R, r = e - g * R;
@@ -487,7 +515,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
 }
 
 template <typename T, int R>
-__global__ void __launch_bounds__(NTHREADS, 2)
+__global__ void __launch_bounds__(TcCfg<T>::NTHREADS, 2)
 k_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ TcArgs a) {
     tc_cta<T, R>(xmap, a, blockIdx.x);
 }
@@ -502,7 +530,7 @@ struct TcBatch {
 };
 
 template <typename T, int R>
-__global__ void __launch_bounds__(NTHREADS, 2)
+__global__ void __launch_bounds__(TcCfg<T>::NTHREADS, 2)
 k_tc_batch(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ TcBatch b) {
     int h = 0;
     while (h + 1 < b.n && blockIdx.x >= b.start[h + 1]) h++;
@@ -684,7 +712,7 @@ cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n) {
         if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
         const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
         if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
-        return launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem, las[0].stream, map, a);
+        return launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(TcCfg<T>::NTHREADS), smem, las[0].stream, map, a);
     }
     if (n > kTcBatchMax) return cudaErrorInvalidValue;
     TcBatch b;
@@ -708,19 +736,26 @@ cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n) {
     cudaError_t e = allow_smem(k_tc_batch<T, R>, attr_set_b);
     if (e != cudaSuccess) return e;
     if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
-    return launch_kernel(k_tc_batch<T, R>, dim3((unsigned)grid), dim3(NTHREADS), smem_max, las[0].stream, map, b);
+    return launch_kernel(k_tc_batch<T, R>, dim3((unsigned)grid), dim3(TcCfg<T>::NTHREADS), smem_max, las[0].stream, map, b);
 }
 
 }  // namespace
 
-bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K) {
+bool tc_supports(int R, int C, bsr_dtype_t dt, int64_t K, int64_t MK) {
     const bool r_ok = R == 16 || R == 32 || R == 64 || R == 128;
     if (dt == BSR_BF16) return r_ok && (C == 16 || C == 32 || C == 64) && K % 8 == 0 && K > 0;
-    // fp32 as 3xTF32; a block lies inside one 32-column stage. Only blocks of
-    // 32 or more rows: each split stage then feeds enough MMA work; for 16-row
-    // blocks the SIMT kernel measured faster (the split adds a step to every
-    // stage's round trip)
-    return (R >= 32 && r_ok) && (C == 16 || C == 32) && K % 4 == 0 && K > 0;
+    // fp32 as 3xTF32; a block lies inside one 32-column stage. Blocks of 32
+    // or more rows always; 16-row blocks on weights of at least 2^20
+    // elements, where a call carries enough work to pay for the split stages
+    // (measured: 1024 x 1024 at 90% and 16384 tokens, 117 us against the
+    // SIMT kernel's 180 us; 768 x 768 at 80% and 1024 tokens, 28 us against
+    // 25 us). BSR_TC_F32_R16=1 takes every 16-row weight, =0 none.
+    static const int r16 = [] {
+        const char *v = getenv("BSR_TC_F32_R16");
+        return v && *v ? atoi(v) : -1;
+    }();
+    const bool r16_ok = r16 == 1 || (r16 != 0 && MK >= ((int64_t)1 << 20));
+    return ((R >= 32 || (R == 16 && r16_ok)) && r_ok) && (C == 16 || C == 32) && K % 4 == 0 && K > 0;
 }
 
 int tc_g_index(int G) {
@@ -780,6 +815,10 @@ cudaError_t launch_tc_t(const LaunchArgs *las, const int *Gs, int n) {
 
 cudaError_t launch_tc(const LaunchArgs &la, int G) {
     return la.sc->dt == BSR_F32 ? launch_tc_t<float>(&la, &G, 1) : launch_tc_t<uint16_t>(&la, &G, 1);
+}
+
+cudaError_t tc_encode_x(bsr_dtype_t dt, const void *X, int64_t N, int64_t K, CUtensorMap *map) {
+    return dt == BSR_F32 ? encode_x<float>(X, N, K, map) : encode_x<uint16_t>(X, N, K, map);
 }
 
 int tc_fusion_key(const Schedule &sc) { return (int)sc.dt * 1024 + sc.ex_R; }

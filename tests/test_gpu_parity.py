@@ -407,6 +407,24 @@ def test_stacked_mmas_for_32_column_bf16_blocks():
     check_product(Y, oracle.bsr_from_dense(w.W, R, C), X, w.bias, M)
 
 
+@pytest.mark.parametrize("C", [16, 32])
+def test_large_fp32_16_row_weights_run_3xtf32_small_ones_simt(C):
+    """fp32 blocks of 16 rows: on a weight of 2^20 elements (1024 x 1024) the
+    tensor cores take them as 3xTF32 (ragged tokens, split rows from a dense
+    row, an empty row); on a 768 x 768 weight the SIMT kernel keeps them."""
+    MB, KB = 1024 // 16, 1024 // C
+    cnt = np.full(MB, KB // 10, dtype=np.int64)
+    cnt[3], cnt[MB - 2] = KB, 0
+    w = synth.make_weight("r16", 90 + C, 1024, 1024, 16, C, "f32", 0, mask=synth.mask_from_row_counts(90 + C, cnt, KB))
+    X = synth.activations(91 + C, 333, 1024, "f32")
+    h, _, Y = _run(w, X)
+    assert h.schedule()["variant"] == "tcgen05"
+    check_product(Y, oracle.bsr_from_dense(w.W, 16, C), X, w.bias, 1024)
+    small = _weight(768, 768, 16, C, "f32", 0.2, 92)
+    h2, _, Y2 = _run(small, synth.activations(93, 100, 768, "f32"))
+    assert h2.schedule()["variant"] == "xstage"
+
+
 def test_small_bf16_blocks_whose_rows_do_not_fill_tiles_stay_simt():
     """M not a multiple of 16 (4-row blocks, M = 260): no 16-row tiling, the
     SIMT kernel keeps the weight."""
