@@ -127,6 +127,7 @@ Schedule::~Schedule() {
         cudaFree(gk.d_wsrc[gi]);
         cudaFree(gk.d_wslot[gi]);
         cudaFree(gk.d_wbase[gi]);
+        cudaFree(gk.d_prog[gi]);
     }
     for (int gi = 0; gi < kTcTaskSizes; gi++) {
         cudaFree(tc.d_rec[gi]);

@@ -19,6 +19,7 @@ constexpr int kGkTmemCols = 512;
 constexpr int kGkTaskSizes = 5;
 constexpr int kGkG[kGkTaskSizes] = {1, 2, 4, 8, 16};
 constexpr int kGkEntryInts = 8;        // ints per (chunk, item) entry
+constexpr int kGkIssuers = 4;          // MMA-issuing threads (one per warp): the issue rate grows with them
 
 // K columns of X per ring stage: 32 KB of fp32 (64 columns) or bf16 (128).
 inline int gk_chunk_cols(bsr_dtype_t dt) { return dt == BSR_F32 ? 64 : 128; }
@@ -35,7 +36,9 @@ bool gk_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 //
 // Record (int32): [ n_items, n_batches, first value byte / 16, record bytes |
 // per chunk c = 0..nchunks: its first batch, padded to 4 | per chunk: its
-// values' byte offset / 16 from the task's first, padded to 4 | per batch
+// values' byte offset / 16 from the task's first, padded to 4 | per chunk:
+// its MMA program's offset / 16 in the programs and its bytes, padded to 4
+// | per batch
 // b = 0..n_batches: its first entry, padded to 4 | per item (row, len, 0, 0)
 // | entries, kGkEntryInts each: (item, first, A column in the batch's
 // buffer, K slices, B byte offset in the chunk's values / 16, blocks, first
@@ -47,6 +50,13 @@ bool gk_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 // (pairs); an item's blocks in a chunk that need more A columns than one
 // buffer holds are split into several entries (pieces). A batch is a run of
 // one chunk's entries whose A columns fit one A buffer.
+//
+// A chunk's MMA program: per batch of the chunk and issuer q the start of
+// its MMAs, then the end (padded to 4 ints), then one 16-byte word per MMA
+// (batch-major, issuer-minor): B offset in the chunk's values / 16,
+// accumulator column, A column in the batch's A buffer (bit 31:
+// accumulate), instruction descriptor. Issuer q owns a contiguous range of
+// the task's items, balanced by work.
 struct GkPlan {
     bool ok = false;
     int64_t off[kGkTaskSizes] = {-1, -1, -1, -1, -1};    // byte offset of G's values in the packed buffer (-1: unusable)
@@ -62,15 +72,18 @@ struct GkPlan {
     std::vector<int32_t> wslot[kGkTaskSizes];          // per packed block slot: (K row of its first column in
                                                        // its entry) | (entry K rows << 16), in packing order
     std::vector<int64_t> wbase[kGkTaskSizes];          // per packed block slot: byte offset of its entry's B operand
+    std::vector<uint32_t> prog[kGkTaskSizes];          // chunk MMA programs of all tasks
+    uint32_t pstage[kGkTaskSizes] = {};                // largest chunk program (bytes)
     int32_t *d_rec[kGkTaskSizes] = {};
     int32_t *d_rec_off[kGkTaskSizes] = {};
     int32_t *d_wsrc[kGkTaskSizes] = {};
     int32_t *d_wslot[kGkTaskSizes] = {};
     int64_t *d_wbase[kGkTaskSizes] = {};
+    uint32_t *d_prog[kGkTaskSizes] = {};
 };
 
 // Shared memory of one CTA with the smallest ring (more than kGkMaxSmem: does not fit).
-size_t gk_smem_bytes(bsr_dtype_t dt, size_t wstage, size_t ibytes, int G, int R);
+size_t gk_smem_bytes(bsr_dtype_t dt, size_t wstage, size_t ibytes, int G, int R);   // wstage: values + program
 // Tensor-memory columns of one A buffer: room for one piece of an entry of
 // at least 32 K columns of fp32 (high and low parts: 64 columns) or 128 of
 // bf16 (pairs: 64 columns), and at least one whole block (C columns). The

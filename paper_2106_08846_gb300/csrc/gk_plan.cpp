@@ -13,6 +13,13 @@ namespace {
 
 int64_t pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
+// Instruction descriptor of the kernel's MMAs: fp32 accumulator, A and B
+// K-major, A/B tf32 (format 2) or bf16 (format 1), N = R, M = 128.
+uint32_t idesc_words(bool f32, int R) {
+    return (1u << 4) | ((f32 ? 2u : 1u) << 7) | ((f32 ? 2u : 1u) << 10) | ((uint32_t)(R >> 3) << 17) |
+           ((uint32_t)(kGkTokens >> 4) << 24);
+}
+
 // Byte offset of chunk column kk in a gk stage at token row 0, before the
 // swizzle: two boxes of 128 token rows x 128 bytes.
 int32_t stage_offset(bsr_dtype_t dt, int64_t kk) {
@@ -41,6 +48,8 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
         pl.wsrc[gi].clear();
         pl.wslot[gi].clear();
         pl.wbase[gi].clear();
+        pl.prog[gi].clear();
+        pl.pstage[gi] = 0;
     }
     if (packed_end < 0 || !gk_supports(sc.R, sc.C, sc.dt, sc.K) || sc.MB == 0 || sc.nnzb == 0) return;
     const bool f32 = sc.dt == BSR_F32;
@@ -90,12 +99,29 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
         int64_t wtotal = 0;   // bytes of packed values of this task size
         std::vector<int32_t> &wsrc = pl.wsrc[gi], &wslot = pl.wslot[gi];
         std::vector<int64_t> &wbase = pl.wbase[gi];
+        std::vector<uint32_t> &prog = pl.prog[gi];
+        size_t pmax = 0;
         std::vector<int64_t> pos;
+        const uint32_t id = idesc_words(f32, (int)R);
         for (int64_t t = 0; t < n_tasks; t++) {
             const std::vector<int64_t> &mem = members[(size_t)t];
             const int g_count = (int)mem.size();
             pos.assign((size_t)g_count, 0);
-            std::vector<int32_t> cb((size_t)nch + 1, 0), cw((size_t)nch + 1, 0), be, entries, clist;
+            std::vector<int32_t> cb((size_t)nch + 1, 0), cw((size_t)nch + 1, 0), cp((size_t)2 * nch, 0), be, entries,
+                clist;
+            // issuer of each item: contiguous ranges balanced by work
+            std::vector<int> owner((size_t)g_count, 0);
+            {
+                int64_t tot = 0, acc = 0;
+                for (int g = 0; g < g_count; g++) tot += work[(size_t)mem[(size_t)g]];
+                for (int g = 0; g < g_count; g++) {
+                    const int64_t w = work[(size_t)mem[(size_t)g]];
+                    owner[(size_t)g] =
+                        tot > 0 ? (int)std::min<int64_t>(kGkIssuers - 1, (2 * acc + w) * kGkIssuers / (2 * tot)) : 0;
+                    acc += w;
+                }
+            }
+            std::vector<std::vector<uint32_t>> words;   // per (batch of the chunk, issuer)
             std::vector<int64_t> cl_of_entry;   // column-list position of each entry (relative)
             std::vector<char> seen((size_t)g_count, 0);
             int64_t cost = 0;
@@ -105,6 +131,7 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
                 cw[(size_t)c] = (int32_t)(wbytes_task / 16);
                 int64_t acol = slot;   // forces a new batch at the chunk's first entry
                 uint32_t boff = 0;
+                words.clear();
                 for (int g = 0; g < g_count; g++) {
                     const int64_t i = mem[(size_t)g];
                     const int32_t p0 = sc.indptr[i] + (int32_t)pos[(size_t)g];
@@ -120,6 +147,25 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
                         if (acol + need > slot) {   // a new batch (a new A buffer)
                             be.push_back((int32_t)(entries.size() / kGkEntryInts));
                             acol = 0;
+                            words.resize(words.size() + kGkIssuers);
+                        }
+                        {
+                            // the entry's MMAs, K slice by K slice: bf16 one,
+                            // fp32 high x high + high x low + low x high (low
+                            // A parts kpad columns on, low B parts kpad R floats on)
+                            std::vector<uint32_t> &wq = words[words.size() - kGkIssuers + (size_t)owner[(size_t)g]];
+                            const uint32_t dcol = (uint32_t)(g * R), bslice = (uint32_t)(R * 32 / 16);
+                            const bool first = !seen[(size_t)g];
+                            for (int64_t q = 0; q < kpad / KS; q++) {
+                                const uint32_t bh = boff / 16 + (uint32_t)q * bslice, ah = (uint32_t)(acol + 8 * q);
+                                const uint32_t acc = (!first || q > 0) ? 0x80000000u : 0u;
+                                wq.insert(wq.end(), {bh, dcol, ah | acc, id});
+                                if (f32) {
+                                    const uint32_t bl = (uint32_t)((boff + kpad * R * 4) / 16) + (uint32_t)q * bslice;
+                                    wq.insert(wq.end(), {bl, dcol, ah | 0x80000000u, id});
+                                    wq.insert(wq.end(), {bh, dcol, (uint32_t)(acol + kpad + 8 * q) | 0x80000000u, id});
+                                }
+                            }
                         }
                         entries.push_back(g);
                         entries.push_back(seen[(size_t)g] ? 0 : 1);
@@ -145,16 +191,33 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
                 }
                 wmax = std::max(wmax, (size_t)boff);
                 wbytes_task += boff;
+                // the chunk's program: starts per (batch, issuer) and the end, then the words
+                if (!words.empty()) {
+                    const size_t at = prog.size(), nstart = words.size() + 1;
+                    prog.resize(at + (size_t)pad4((int64_t)nstart), 0u);
+                    uint32_t n = 0;
+                    for (size_t k = 0; k < words.size(); k++) {
+                        prog[at + k] = n;
+                        n += (uint32_t)(words[k].size() / 4);
+                    }
+                    prog[at + words.size()] = n;
+                    for (const auto &w : words) prog.insert(prog.end(), w.begin(), w.end());
+                    cp[(size_t)(2 * c)] = (int32_t)(at / 4);
+                    cp[(size_t)(2 * c + 1)] = (int32_t)((prog.size() - at) * 4);
+                    pmax = std::max(pmax, (prog.size() - at) * 4);
+                }
             }
             const int n_batches = (int)be.size();
             cb[(size_t)nch] = n_batches;
             cw[(size_t)nch] = (int32_t)(wbytes_task / 16);
             be.push_back((int32_t)(entries.size() / kGkEntryInts));
             const int64_t n_ent = (int64_t)cl_of_entry.size();
-            // [ header | chunk batches | chunk W offsets | batch entries | items | entries | column list ]
+            // [ header | chunk batches | chunk W offsets | chunk programs | batch entries | items | entries
+            //   | column list ]
             const int64_t head = (int64_t)rec.size();
             roff.push_back((int32_t)head);
-            const int64_t cb_at = 4, cw_at = cb_at + pad4(nch + 1), be_at = cw_at + pad4(nch + 1);
+            const int64_t cb_at = 4, cw_at = cb_at + pad4(nch + 1), cp_at = cw_at + pad4(nch + 1);
+            const int64_t be_at = cp_at + pad4(2 * nch);
             const int64_t items_at = be_at + pad4(n_batches + 1), ent_at = items_at + 4 * g_count;
             const int64_t cl_at = ent_at + kGkEntryInts * n_ent;
             const int64_t total_ints = pad4(cl_at + (int64_t)clist.size());
@@ -166,6 +229,7 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
             r[3] = (int32_t)(total_ints * 4);
             std::copy(cb.begin(), cb.end(), r + cb_at);
             std::copy(cw.begin(), cw.end(), r + cw_at);
+            std::copy(cp.begin(), cp.end(), r + cp_at);
             std::copy(be.begin(), be.end(), r + be_at);
             for (int g = 0; g < g_count; g++) {
                 const int64_t i = mem[(size_t)g];
@@ -181,17 +245,20 @@ void plan_gk(Schedule &sc, int64_t packed_end) {
         }
         pl.n_tasks[gi] = (int)n_tasks;
         pl.wstage[gi] = (uint32_t)((wmax + 15) & ~size_t(15));
+        pl.pstage[gi] = (uint32_t)((pmax + 15) & ~size_t(15));
         pl.ibytes[gi] = (uint32_t)((imax + 15) & ~size_t(15));
         pl.acols[gi] = (uint32_t)slot;
         pl.cost_max[gi] = cost_max;
-        const bool fits = gk_smem_bytes(sc.dt, pl.wstage[gi], pl.ibytes[gi], G, sc.R) <= (size_t)kGkMaxSmem &&
-                          (int64_t)rec.size() < INT32_MAX && wtotal / 16 < INT32_MAX;
+        const bool fits = gk_smem_bytes(sc.dt, pl.wstage[gi] + pl.pstage[gi], pl.ibytes[gi], G, sc.R) <=
+                              (size_t)kGkMaxSmem &&
+                          (int64_t)rec.size() < INT32_MAX && wtotal / 16 < INT32_MAX && prog.size() / 4 < INT32_MAX;
         if (!fits) {
             rec.clear();
             roff.clear();
             wsrc.clear();
             wslot.clear();
             wbase.clear();
+            prog.clear();
             continue;
         }
         pl.off[gi] = end;

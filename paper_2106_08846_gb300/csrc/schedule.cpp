@@ -547,7 +547,8 @@ bsr_status_t build_schedule(Schedule &sc) {
             upload(&sc.gk.d_rec_off[gi], sc.gk.rec_off[gi]) != cudaSuccess ||
             upload(&sc.gk.d_wsrc[gi], sc.gk.wsrc[gi]) != cudaSuccess ||
             upload(&sc.gk.d_wslot[gi], sc.gk.wslot[gi]) != cudaSuccess ||
-            upload(&sc.gk.d_wbase[gi], sc.gk.wbase[gi]) != cudaSuccess) {
+            upload(&sc.gk.d_wbase[gi], sc.gk.wbase[gi]) != cudaSuccess ||
+            upload(&sc.gk.d_prog[gi], sc.gk.prog[gi]) != cudaSuccess) {
             cudaGetLastError();
             return BSR_ERR_ALLOC;
         }

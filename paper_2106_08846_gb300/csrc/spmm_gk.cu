@@ -21,23 +21,29 @@
 //                         one per item, over that item's gathered K,
 //                         zero-padded to the MMA's K), through a ring of
 //                         stages that keeps streaming across units.
-//   warp 1 (one thread)  owns the tensor memory and issues the MMAs: per
-//                         batch of entries (pieces of a chunk's items, as
-//                         many as fill one of up to eight A buffers, so the
-//                         gather runs several batches ahead of the MMAs'
-//                         completion) and K slice, M = 128, N = R,
-//                         K = 8 (tf32; three per slice) or 16 (bf16), A from
+//   warps 1..4 (lane 0)  issue the MMAs (warp 1 also owns the tensor
+//                         memory): one thread issues an MMA no faster than
+//                         every 40-100 ns, so four issuers each run the
+//                         MMAs of a contiguous, work-balanced range of the
+//                         task's items, from a program built at create time
+//                         and loaded beside each chunk's block values (one
+//                         16-byte word per MMA: no decoding between MMAs).
+//                         Per batch of entries (pieces of a chunk's items,
+//                         as many as fill one of up to eight A buffers, so
+//                         the gather runs several batches ahead of the MMAs'
+//                         completion) and K slice: M = 128, N = R, K = 8
+//                         (tf32; three per slice) or 16 (bf16), A from
 //                         tensor memory, B from shared memory; commits free
 //                         the A buffer, the stage and, per unit, hand the
 //                         accumulators to the epilogue.
-//   warps 2..9           gather, two groups of four warps (one per 32 lanes)
+//   warps 5..12          gather, two groups of four warps (one per 32 lanes)
 //                         taking alternate batches, so two batches are in
 //                         flight: thread t (token t, tensor-memory lane t) reads its
 //                         token's values of each entry's kept columns from
 //                         the stage, splits fp32 into tf32 high and low parts,
 //                         and stores them with tcgen05.st into the batch's A
 //                         buffer (zeros pad each entry's K).
-//   warps 10..13         epilogue: each reads its 32 lanes of the
+//   warps 13..16         epilogue: each reads its 32 lanes of the
 //                         accumulators, adds the bias, turns the tile around
 //                         through shared memory and stores whole row segments
 //                         of Y, then frees the accumulators for the next unit
@@ -66,9 +72,10 @@ namespace {
 constexpr int TN = kGkTokens;
 constexpr int NS_MAX = kGkStages;
 constexpr int NA_MAX = kGkASlotsMax;
+constexpr int NISS = kGkIssuers;       // MMA-issuing warps (lane 0 of each)
 constexpr int NGW = 8;                 // gather warps: two groups of one warp per tensor-memory lane quarter
 constexpr int NEW = 4;                 // epilogue warps: one per lane quarter
-constexpr int NWARPS = 2 + NGW + NEW;
+constexpr int NWARPS = 1 + NISS + NGW + NEW;
 constexpr int NTHREADS = NWARPS * 32;
 constexpr uint32_t kStageBytes = TN * 256;   // two 128-byte-row boxes of 128 tokens
 constexpr uint64_t kDrainNs = 200000000ull;
@@ -79,7 +86,8 @@ struct GkArgs {
     const int32_t *rec;       // task records
     const int32_t *rec_off;   // per task: record offset (ints)
     const unsigned char *wpk; // packed block values of this task size
-    uint32_t wstage;          // bytes of one W stage
+    const uint4 *prog;        // chunk MMA programs of this task size
+    uint32_t wstage, wslot;   // bytes of a chunk's values (most), of one W stage (values + program)
     uint32_t acols;           // tensor-memory columns of one A buffer
     const float *bias;
     void *Y;
@@ -292,7 +300,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
     unsigned char *base =
         reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(base + a.bar_off);
-    uint64_t *empty = full + NS_MAX;   // the gather warps + the MMA commit
+    uint64_t *empty = full + NS_MAX;   // the gather warps + every issuer's MMA commit
     uint64_t *afull = empty + NS_MAX;  // A buffer written (one gather group)
     uint64_t *aempty = afull + NA_MAX; // A buffer consumed (MMA commit)
     uint64_t *accf = aempty + NA_MAX;  // a unit's MMAs completed (MMA commit)
@@ -308,7 +316,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
     const int64_t n_tiles = (a.N + TN - 1) / TN;
     const int64_t units = n_tiles * a.n_tasks, P = gridDim.x;
     const int64_t ub = units * (int64_t)blockIdx.x / P, ue = units * ((int64_t)blockIdx.x + 1) / P;
-    const int cb_at = 4, cw_at = 4 + pad4(nch + 1), be_at = cw_at + pad4(nch + 1);
+    const int cb_at = 4, cw_at = 4 + pad4(nch + 1), cp_at = cw_at + pad4(nch + 1), be_at = cp_at + pad4(2 * nch);
     auto rec_s = [&](int j) { return reinterpret_cast<int32_t *>(base + a.rec_smem + (j & 1) * a.rec_bytes); };
     auto bias_s = [&](int j) { return reinterpret_cast<float *>(base + a.bias_off) + (j & 1) * a.G * R; };
     auto last_of_task = [&](int64_t u) { return u + 1 == ue || (u + 1) / n_tiles != u / n_tiles; };
@@ -316,19 +324,19 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS_MAX; s++) {
             ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], NGW + 1);
+            ptx::mbar_init(&empty[s], NGW + NISS);
         }
         for (int s = 0; s < NA_MAX; s++) {
             ptx::mbar_init(&afull[s], 4);
-            ptx::mbar_init(&aempty[s], 1);
+            ptx::mbar_init(&aempty[s], NISS);
         }
-        ptx::mbar_init(accf, 1);
+        ptx::mbar_init(accf, NISS);
         ptx::mbar_init(acce, NEW);
         for (int r = 0; r < 2; r++) {
             ptx::mbar_init(&rbar[r], 1);
-            ptx::mbar_init(&rfree[r], 1 + NGW + NEW);
+            ptx::mbar_init(&rfree[r], NISS + NGW + NEW);
         }
-        ptx::mbar_init(done, 1);
+        ptx::mbar_init(done, NISS);
         misc[0] = 0;
         ptx::fence_barrier_init();
     }
@@ -388,12 +396,15 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                         stalled = k++;
                         continue;
                     }
+                    // the X chunk, the chunk's block values and, after them, its MMA program
                     const uint32_t w0 = (uint32_t)I[cw_at + c] * 16u, wbytes = (uint32_t)I[cw_at + c + 1] * 16u - w0;
+                    const uint32_t pbytes = (uint32_t)I[cp_at + 2 * c + 1];
                     constexpr int KC = F32 ? 64 : 128, BOXC = F32 ? 32 : 64;
-                    ptx::mbar_arrive_expect_tx(&full[s], kStageBytes + wbytes);
+                    ptx::mbar_arrive_expect_tx(&full[s], kStageBytes + wbytes + pbytes);
                     ptx::tma_load_2d(base + s * kStageBytes, &xmap, c * KC, n0, &full[s]);
                     ptx::tma_load_2d(base + s * kStageBytes + kStageBytes / 2, &xmap, c * KC + BOXC, n0, &full[s]);
-                    ptx::bulk_load(W_s + s * a.wstage, a.wpk + wfirst + w0, wbytes, &full[s]);
+                    ptx::bulk_load(W_s + s * a.wslot, a.wpk + wfirst + w0, wbytes, &full[s]);
+                    ptx::bulk_load(W_s + s * a.wslot + a.wstage, a.prog + I[cp_at + 2 * c], pbytes, &full[s]);
                     k++;
                 }
             }
@@ -406,11 +417,11 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                 if (d != stalled) ptx::mbar_wait_bounded(&full[d % ns], (uint32_t)(d / ns) & 1, kDrainNs);
             ptx::mbar_wait_bounded(&rbar[j & 1], (j >> 1) & 1, kDrainNs);
         }
-    } else if (warp == 1) {
-        // ---------------- MMA issuer
+    } else if (warp <= NISS) {
+        // ---------------- MMA issuers: lane 0 of warps 1..NISS, each running
+        // its part of every batch's program (its items' MMAs), one word per MMA
         if (lane == 0) {
-            constexpr uint32_t id = idesc(F32, TN, R);
-            constexpr uint32_t bslice = (uint32_t)R * 32u;   // bytes of one K slice of B
+            const int q = warp - 1;
             bool ok = true;
             int j = -1;
             int64_t task = -1, k = 0, kb = 0, ui = 0;
@@ -421,7 +432,6 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                     if (!ptx::mbar_wait_bounded(&rbar[j & 1], (j >> 1) & 1, a.wait_ns)) { ok = false; break; }
                 }
                 const int32_t *I = rec_s(j);
-                const int32_t *ent = I + be_at + pad4(I[1] + 1) + 4 * I[0];
                 // the epilogue has read the previous unit's accumulators
                 if (ui > 0 && !ptx::mbar_wait_bounded(acce, (uint32_t)(ui - 1) & 1, a.wait_ns)) { ok = false; break; }
                 tc_fence_after();
@@ -433,7 +443,10 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                         ok = false;
                         break;
                     }
-                    const uint32_t wsb = ptx::smem_addr(W_s + s * a.wstage);
+                    const unsigned char *slot = W_s + s * a.wslot;
+                    const uint64_t bd0 = umma_desc(ptx::smem_addr(slot), 128, 256);
+                    const int32_t *hdr = reinterpret_cast<const int32_t *>(slot + a.wstage);
+                    const uint4 *pw = reinterpret_cast<const uint4 *>(hdr + pad4((b1 - b0) * NISS + 1));
                     for (int b = b0; b < b1; b++) {
                         const int sl = (int)(kb % na);
                         if (!ptx::mbar_wait_bounded(&afull[sl], (uint32_t)(kb / na) & 1, a.wait_ns) || aborted(misc)) {
@@ -442,30 +455,18 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                         }
                         tc_fence_after();
                         const uint32_t ab = abase + (uint32_t)sl * a.acols;
-                        for (int e = I[be_at + b]; e < I[be_at + b + 1]; e++) {
-                            const int32_t *en = ent + EI * e;
-                            const uint32_t d = tmem + (uint32_t)(en[0] * R);
-                            const uint32_t first = (uint32_t)en[1], acol = ab + (uint32_t)en[2];
-                            const int nsl = en[3];
-                            const uint32_t bb = wsb + (uint32_t)en[4] * 16u;
-                            if constexpr (F32) {
-                                const int kpad = nsl * 8;
-                                const uint32_t blo = bb + (uint32_t)kpad * R * 4u;
-                                for (int q = 0; q < nsl; q++) {
-                                    const uint64_t bh = umma_desc(bb + q * bslice, 128, 256),
-                                                   bl = umma_desc(blo + q * bslice, 128, 256);
-                                    const uint32_t ah = acol + 8u * q, al = acol + (uint32_t)kpad + 8u * q;
-                                    mma_ts<true>(d, ah, bh, id, (first == 0u) | (q > 0));
-                                    mma_ts<true>(d, ah, bl, id, 1u);
-                                    mma_ts<true>(d, al, bh, id, 1u);
-                                }
-                            } else {
-                                for (int q = 0; q < nsl; q++)
-                                    mma_ts<false>(d, acol + 8u * q, umma_desc(bb + q * bslice, 128, 256), id,
-                                                  (first == 0u) | (q > 0));
-                            }
+                        const int i1 = hdr[(b - b0) * NISS + q + 1];
+                        int i = hdr[(b - b0) * NISS + q];
+                        for (; i + 2 <= i1; i += 2) {   // two words loaded ahead of their MMAs
+                            const uint4 w0 = pw[i], w1 = pw[i + 1];
+                            mma_ts<F32>(tmem + w0.y, ab + (w0.z & 0x7fffffffu), bd0 + w0.x, w0.w, w0.z >> 31);
+                            mma_ts<F32>(tmem + w1.y, ab + (w1.z & 0x7fffffffu), bd0 + w1.x, w1.w, w1.z >> 31);
                         }
-                        mma_commit(&aempty[sl]);   // the A buffer is free once these MMAs completed
+                        if (i < i1) {
+                            const uint4 w0 = pw[i];
+                            mma_ts<F32>(tmem + w0.y, ab + (w0.z & 0x7fffffffu), bd0 + w0.x, w0.w, w0.z >> 31);
+                        }
+                        mma_commit(&aempty[sl]);   // the A buffer is free once every issuer's MMAs completed
                         kb++;
                     }
                     if (!ok) break;
@@ -480,15 +481,14 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                 set_status(a.status, DEV_TIMEOUT);
                 atomicExch(&misc[0], 1);
             }
-            mma_commit(done);   // every MMA issued above completes before `done`
-            // the tensor memory is freed below: wait (this thread alone, so the
-            // warp's other lanes never spin beside the issuing one) for them
-            if (!ptx::mbar_wait_bounded(done, 0, kDrainNs)) set_status(a.status, DEV_TIMEOUT);
+            mma_commit(done);   // every MMA this issuer issued completes before its arrival
+            // the tensor memory is freed below: one thread waits for every issuer's MMAs
+            if (warp == 1 && !ptx::mbar_wait_bounded(done, 0, kDrainNs)) set_status(a.status, DEV_TIMEOUT);
         }
-    } else if (warp < 2 + NGW) {
-        // ---------------- gather; lane quarter = warp % 4, group (warps 2..5
-        // or 6..9) takes the batches of its parity
-        const int q = warp & 3, grp = (warp - 2) >> 2;
+    } else if (warp <= NISS + NGW) {
+        // ---------------- gather; lane quarter = warp % 4, group (the first
+        // or the second four gather warps) takes the batches of its parity
+        const int q = warp & 3, grp = (warp - 1 - NISS) >> 2;
         const int t = 32 * q + lane;   // token row in the tile = tensor-memory lane
         const uint32_t sw = (uint32_t)(t & 7) << 4;
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
@@ -544,7 +544,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
         // ---------------- epilogue; lane quarter = warp % 4
         const int q = warp & 3;
         const int t = 32 * q + lane;
-        const int et = threadIdx.x - 32 * (2 + NGW);   // 0..127
+        const int et = threadIdx.x - 32 * (1 + NISS + NGW);   // 0..127
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
         ptx::pdl_wait();   // the bias and Y may be an earlier kernel's
         bool ok = true;
@@ -575,7 +575,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
             // this warp's staging tile (16-byte groups XOR-swizzled by row), then
             // lanes re-read it as (row, 8-column group) pairs and store whole row
             // segments: 8 rows x 4 groups per instruction
-            float *stg = reinterpret_cast<float *>(base + a.stg_off) + (warp - 2 - NGW) * 32 * 32;
+            float *stg = reinterpret_cast<float *>(base + a.stg_off) + (warp - 1 - NISS - NGW) * 32 * 32;
             const uint32_t stg_row = ptx::smem_addr(stg) + (uint32_t)lane * 128u;
             const int64_t row0 = (u % n_tiles) * TN + 32 * q;   // the warp's first token
             for (int g = 0; g < I[0]; g++) {
@@ -777,6 +777,9 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.rec_off = pl.d_rec_off[gi];
     a.wpk = static_cast<const unsigned char *>(la.data) + pl.off[gi];
     a.wstage = pl.wstage[gi];
+    a.wslot = pl.wstage[gi] + pl.pstage[gi];
+    a.prog = reinterpret_cast<const uint4 *>(pl.d_prog[gi]);
+    if (!a.prog) return cudaErrorInvalidConfiguration;
     a.acols = pl.acols[gi];
     a.na = gk_slots(R, sc.C, sizeof(T) == 4, G);
     a.bias = la.bias;
@@ -790,7 +793,7 @@ cudaError_t launch_r(const LaunchArgs &la, int G) {
     a.wait_ns = la.wait_ns;
     a.stall_chunk = la.stall_chunk;
     uint32_t smem = 0;
-    for (int ns = NS_MAX; ns >= 2 && !smem; ns--) smem = layout(ns, a.wstage, pl.ibytes[gi], G, R, &a);
+    for (int ns = NS_MAX; ns >= 2 && !smem; ns--) smem = layout(ns, a.wslot, pl.ibytes[gi], G, R, &a);
     if (!smem || a.na < 2 || (uint32_t)(G * R) + (uint32_t)a.na * a.acols > (uint32_t)kGkTmemCols)
         return cudaErrorInvalidConfiguration;
     static std::atomic<uint64_t> attr_set{0};
