@@ -464,12 +464,17 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
 #pragma unroll
                 for (int j = 0; j < 16; j++) v[j] = len > 0 ? __uint_as_float(h < 32 ? r0[h + j] : r1[h - 32 + j]) : 0.f;
                 if (slot < 0) {
+                    // staged rows in the Y map's swizzled order (64-byte fp32 rows:
+                    // 16-byte group j of row t at j ^ ((t / 2) % 4); 32-byte bf16
+                    // rows: j ^ ((t / 4) % 2)), so a warp's stores spread over
+                    // all banks; the TMA store writes Y's rows in plain order
                     unsigned char *row = buf + (h / 16) * kGroupBytes + t * 16 * (int)sizeof(T);
                     if constexpr (F32) {
                         float4 *dst = reinterpret_cast<float4 *>(row);
+                        const int sw = (t >> 1) & 3;
 #pragma unroll
                         for (int j = 0; j < 4; j++)
-                            dst[j] = make_float4(v[4 * j] + B_s[col + 4 * j], v[4 * j + 1] + B_s[col + 4 * j + 1],
+                            dst[j ^ sw] = make_float4(v[4 * j] + B_s[col + 4 * j], v[4 * j + 1] + B_s[col + 4 * j + 1],
                                                  v[4 * j + 2] + B_s[col + 4 * j + 2], v[4 * j + 3] + B_s[col + 4 * j + 3]);
                     } else {
                         uint32_t pk[8];
@@ -480,8 +485,9 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                             pk[j] = (uint32_t)from_f32<uint16_t>(lo) | ((uint32_t)from_f32<uint16_t>(hi) << 16);
                         }
                         uint4 *dst = reinterpret_cast<uint4 *>(row);
-                        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                        const int sw = (t >> 2) & 1;
+                        dst[sw] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        dst[1 ^ sw] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                     }
                 } else if (n < a.N) {
                     float4 *dst = reinterpret_cast<float4 *>(a.ws + ((int64_t)slot * a.N + n) * R + hr);
@@ -608,7 +614,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // Y [N, M] for the epilogue's TMA stores: boxes of 16 columns x 128 token rows,
-// no swizzle (the staged rows are plain row-major).
+// with the swizzle of the row size (64 bytes fp32, 32 bytes bf16) in which
+// the epilogue stages them.
 template <typename T>
 cudaError_t encode_y(void *Y, int64_t N, int64_t M, CUtensorMap *map) {
     auto enc = encode_fn();
@@ -618,7 +625,8 @@ cudaError_t encode_y(void *Y, int64_t N, int64_t M, CUtensorMap *map) {
     const cuuint32_t box[2] = {16, (cuuint32_t)TN};
     const cuuint32_t estr[2] = {1, 1};
     if (enc(map, sizeof(T) == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, Y, dims,
-            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            sizeof(T) == 4 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B,
             CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return cudaErrorInvalidValue;
     return cudaSuccess;
