@@ -64,6 +64,7 @@
 #include "gk.h"
 #include "launch.cuh"
 #include "ptx.cuh"
+#include "tcgen05.cuh"
 
 namespace bsr {
 
@@ -98,66 +99,6 @@ struct GkArgs {
     uint64_t wait_ns;
     int stall_chunk;              // test hook: this chunk of each CTA's first unit is never loaded (-1: none)
 };
-
-__device__ __forceinline__ uint64_t umma_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
-    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
-           ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | (1ull << 46);
-}
-// Instruction descriptors: fp32 accumulator, A and B K-major; A/B format 2
-// (tf32) or 1 (bf16); N / 8 and M / 16.
-__host__ __device__ constexpr uint32_t idesc(bool f32, int M, int N) {
-    return (1u << 4) | ((f32 ? 2u : 1u) << 7) | ((f32 ? 2u : 1u) << 10) | ((uint32_t)(N >> 3) << 17) |
-           ((uint32_t)(M >> 4) << 24);
-}
-
-// D (tensor memory) (+)= A (tensor memory) x B (shared-memory descriptor)
-template <bool F32>
-__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t id, uint32_t acc) {
-    if constexpr (F32)
-        asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
-                     "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}"
-                     ::"r"(d), "r"(a), "l"(b), "r"(id), "r"(acc));
-    else
-        asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
-                     "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}"
-                     ::"r"(d), "r"(a), "l"(b), "r"(id), "r"(acc));
-}
-
-__device__ __forceinline__ void mma_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                     ptx::smem_addr(bar))
-                 : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// 8 32-bit columns of this thread's lane (warp-wide, same column for all lanes)
-__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
-                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
-                 : "memory");
-}
-__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-
-// 32 lanes x 32 columns of fp32 from tensor memory (no wait).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-}
-// 16 columns
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-}
 
 __device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(status, DEV_OK, code); }
 __device__ __forceinline__ bool aborted(const int *flag) { return *reinterpret_cast<const volatile int *>(flag) != 0; }
@@ -240,8 +181,8 @@ __device__ __forceinline__ void gather_entry(uint32_t row, uint32_t sw, const in
                 hi[i] = __float_as_uint(h);
                 lo[i] = __float_as_uint(v[i] - h);
             }
-            tmem_st8(col + (uint32_t)k0, hi);
-            tmem_st8(col + (uint32_t)(kpad + k0), lo);
+            tc5::st8(col + (uint32_t)k0, hi);
+            tc5::st8(col + (uint32_t)(kpad + k0), lo);
         }
     } else {
         for (int k0 = 0; k0 < kpad; k0 += 16) {
@@ -285,7 +226,7 @@ __device__ __forceinline__ void gather_entry(uint32_t row, uint32_t sw, const in
                     }
                 }
             }
-            tmem_st8(col + (uint32_t)(k0 / 2), p);
+            tc5::st8(col + (uint32_t)(k0 / 2), p);
         }
     }
 }
@@ -340,16 +281,10 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
         misc[0] = 0;
         ptx::fence_barrier_init();
     }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         ptx::smem_addr(&misc[1])),
-                     "r"(kGkTmemCols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    tc_fence_before();
+    if (warp == 1) tc5::alloc(reinterpret_cast<uint32_t *>(&misc[1]), kGkTmemCols);
+    tc5::fence_before();
     __syncthreads();
-    tc_fence_after();
+    tc5::fence_after();
     const uint32_t tmem = (uint32_t)misc[1];
     const uint32_t abase = tmem + (uint32_t)(a.G * R);   // A buffers after the accumulators
 
@@ -434,7 +369,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                 const int32_t *I = rec_s(j);
                 // the epilogue has read the previous unit's accumulators
                 if (ui > 0 && !ptx::mbar_wait_bounded(acce, (uint32_t)(ui - 1) & 1, a.wait_ns)) { ok = false; break; }
-                tc_fence_after();
+                tc5::fence_after();
                 for (int c = 0; ok && c < nch; c++) {
                     const int b0 = I[cb_at + c], b1 = I[cb_at + c + 1];
                     if (b0 == b1) continue;
@@ -444,7 +379,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                         break;
                     }
                     const unsigned char *slot = W_s + s * a.wslot;
-                    const uint64_t bd0 = umma_desc(ptx::smem_addr(slot), 128, 256);
+                    const uint64_t bd0 = tc5::desc(ptx::smem_addr(slot), 128, 256);
                     const int32_t *hdr = reinterpret_cast<const int32_t *>(slot + a.wstage);
                     const uint4 *pw = reinterpret_cast<const uint4 *>(hdr + pad4((b1 - b0) * NISS + 1));
                     for (int b = b0; b < b1; b++) {
@@ -453,35 +388,35 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                             ok = false;
                             break;
                         }
-                        tc_fence_after();
+                        tc5::fence_after();
                         const uint32_t ab = abase + (uint32_t)sl * a.acols;
                         const int i1 = hdr[(b - b0) * NISS + q + 1];
                         int i = hdr[(b - b0) * NISS + q];
                         for (; i + 2 <= i1; i += 2) {   // two words loaded ahead of their MMAs
                             const uint4 w0 = pw[i], w1 = pw[i + 1];
-                            mma_ts<F32>(tmem + w0.y, ab + (w0.z & 0x7fffffffu), bd0 + w0.x, w0.w, w0.z >> 31);
-                            mma_ts<F32>(tmem + w1.y, ab + (w1.z & 0x7fffffffu), bd0 + w1.x, w1.w, w1.z >> 31);
+                            tc5::mma_ts<F32>(tmem + w0.y, ab + (w0.z & 0x7fffffffu), bd0 + w0.x, w0.w, w0.z >> 31);
+                            tc5::mma_ts<F32>(tmem + w1.y, ab + (w1.z & 0x7fffffffu), bd0 + w1.x, w1.w, w1.z >> 31);
                         }
                         if (i < i1) {
                             const uint4 w0 = pw[i];
-                            mma_ts<F32>(tmem + w0.y, ab + (w0.z & 0x7fffffffu), bd0 + w0.x, w0.w, w0.z >> 31);
+                            tc5::mma_ts<F32>(tmem + w0.y, ab + (w0.z & 0x7fffffffu), bd0 + w0.x, w0.w, w0.z >> 31);
                         }
-                        mma_commit(&aempty[sl]);   // the A buffer is free once every issuer's MMAs completed
+                        tc5::commit(&aempty[sl]);   // the A buffer is free once every issuer's MMAs completed
                         kb++;
                     }
                     if (!ok) break;
-                    mma_commit(&empty[s]);   // and so are the stage's block values
+                    tc5::commit(&empty[s]);   // and so are the stage's block values
                     k++;
                 }
                 if (!ok) break;
-                mma_commit(accf);   // the unit's accumulators are complete
+                tc5::commit(accf);   // the unit's accumulators are complete
                 if (last_of_task(u)) ptx::mbar_arrive(&rfree[j & 1]);
             }
             if (!ok) {
                 set_status(a.status, DEV_TIMEOUT);
                 atomicExch(&misc[0], 1);
             }
-            mma_commit(done);   // every MMA this issuer issued completes before its arrival
+            tc5::commit(done);   // every MMA this issuer issued completes before its arrival
             // the tensor memory is freed below: one thread waits for every issuer's MMAs
             if (warp == 1 && !ptx::mbar_wait_bounded(done, 0, kDrainNs)) set_status(a.status, DEV_TIMEOUT);
         }
@@ -519,14 +454,14 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                     bool free = true;
                     if (kb >= na) free = ptx::mbar_wait_bounded(&aempty[sl], (uint32_t)((kb / na) - 1) & 1, a.wait_ns);
                     if (!__all_sync(0xffffffffu, free && !aborted(misc))) { ok = false; break; }
-                    tc_fence_after();
+                    tc5::fence_after();
                     const uint32_t ab = abase + (uint32_t)sl * a.acols + lane_off;
                     for (int e = I[be_at + b]; e < I[be_at + b + 1]; e++) {
                         const int32_t *en = ent + EI * e;
                         gather_entry<F32>(row, sw, I + en[6], en[5], lc, en[3] * KS, ab + (uint32_t)en[2]);
                     }
-                    tmem_st_wait();
-                    tc_fence_before();
+                    tc5::st_wait();
+                    tc5::fence_before();
                     __syncwarp();
                     if (lane == 0) ptx::mbar_arrive(&afull[sl]);
                 }
@@ -543,7 +478,6 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
     } else {
         // ---------------- epilogue; lane quarter = warp % 4
         const int q = warp & 3;
-        const int t = 32 * q + lane;
         const int et = threadIdx.x - 32 * (1 + NISS + NGW);   // 0..127
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
         ptx::pdl_wait();   // the bias and Y may be an earlier kernel's
@@ -570,7 +504,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
             const uint64_t limit = a.wait_ns * (uint64_t)(nch + 2);
             const bool got = ptx::mbar_wait_bounded(accf, (uint32_t)ui & 1, limit) && !aborted(misc);
             if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
-            tc_fence_after();
+            tc5::fence_after();
             // per item and 32-column group: each lane's row of the tile into
             // this warp's staging tile (16-byte groups XOR-swizzled by row), then
             // lanes re-read it as (row, 8-column group) pairs and store whole row
@@ -585,14 +519,14 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                     constexpr int W = R >= 32 ? 32 : R;
                     uint32_t r[32];
                     if constexpr (W == 32) {
-                        tmem_ld32(tmem + lane_off + (uint32_t)(g * R + c0), r);
+                        tc5::ld32(tmem + lane_off + (uint32_t)(g * R + c0), r);
                     } else {
                         uint32_t r16[16];
-                        tmem_ld16(tmem + lane_off + (uint32_t)(g * R + c0), r16);
+                        tc5::ld16(tmem + lane_off + (uint32_t)(g * R + c0), r16);
 #pragma unroll
                         for (int i = 0; i < 16; i++) r[i] = r16[i];
                     }
-                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                    tc5::ld_wait();
                     const float *bs = B + g * R + c0;
 #pragma unroll
                     for (int c4 = 0; c4 < W / 4; c4++) {
@@ -638,7 +572,7 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
                     __syncwarp();   // the staging tile is free again
                 }
             }
-            tc_fence_before();
+            tc5::fence_before();
             __syncwarp();
             if (lane == 0) {
                 ptx::mbar_arrive(acce);   // the accumulators may be overwritten
@@ -652,11 +586,11 @@ k_gk(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ GkArgs a)
     }
     // ---------------- teardown: every MMA issued completed (the issuer waited
     // for them), then free the tensor memory
-    tc_fence_before();
+    tc5::fence_before();
     __syncthreads();
     if (warp == 1) {
-        tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kGkTmemCols) : "memory");
+        tc5::fence_after();
+        tc5::dealloc(tmem, kGkTmemCols);
     }
 }
 

@@ -50,6 +50,7 @@
 #include "launch.cuh"
 #include "ptx.cuh"
 #include "tc.h"
+#include "tcgen05.cuh"
 
 namespace bsr {
 
@@ -87,40 +88,6 @@ struct TcArgs {
     int stall_chunk;
 };
 
-// ---- tcgen05 / UMMA wrappers
-
-// Shared-memory matrix descriptor: start address, leading and stride byte
-// offsets (16-byte units), descriptor version 1, layout (0: no swizzle,
-// 2: 128-byte swizzle).
-__device__ __forceinline__ uint64_t umma_desc(uint32_t addr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
-    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
-           ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | (1ull << 46) | ((uint64_t)layout << 61);
-}
-
-// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, both K-major.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc));
-}
-
-// Instruction descriptor of kind::tf32: tf32 A and B (format 2), fp32 D, both K-major.
-__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
-    return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
-
-__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(acc));
-}
-
 // fp32 -> (high, low) with high = x with the low 13 mantissa bits cleared
 // (a tf32 value) and low = x - high, exact in fp32.
 __device__ __forceinline__ float4 tf32_high(float4 v) {
@@ -128,32 +95,10 @@ __device__ __forceinline__ float4 tf32_high(float4 v) {
                        __uint_as_float(__float_as_uint(v.z) & 0xffffe000u), __uint_as_float(__float_as_uint(v.w) & 0xffffe000u));
 }
 
-// The mbarrier arrives once every MMA this thread issued so far completed.
-__device__ __forceinline__ void mma_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                     ptx::smem_addr(bar))
-                 : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
 __device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(status, DEV_OK, code); }
 __device__ __forceinline__ bool aborted(const int *flag) { return *reinterpret_cast<const volatile int *>(flag) != 0; }
 
 __device__ __forceinline__ int pad4(int n) { return (n + 3) & ~3; }
-
-// 32 lanes x 32 columns of fp32 from tensor memory (no wait).
-__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-}
 
 // One CTA of the product described by `a`; `cta` is its index in that
 // product's grid (tile-fastest).
@@ -207,16 +152,10 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
         itab[6 * g + 4] = 0;
         itab[6 * g + 5] = it.z - it.y;
     }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         ptx::smem_addr(&misc[1])),
-                     "r"(a.tmem_cols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    tc_fence_before();
+    if (warp == 1) tc5::alloc(reinterpret_cast<uint32_t *>(&misc[1]), a.tmem_cols);
+    tc5::fence_before();
     __syncthreads();
-    tc_fence_after();
+    tc5::fence_after();
     const uint32_t tmem = (uint32_t)misc[1];
     const uint32_t wblock = (uint32_t)R * C * (F32 ? 8 : 2);   // bytes of one block's B operand(s)
 
@@ -300,13 +239,13 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                     ok = false;
                     break;
                 }
-                tc_fence_after();
+                tc5::fence_after();
                 const uint32_t stage = ptx::smem_addr(base + s * kStageBytes);
                 const uint32_t w_stage = ptx::smem_addr(W_s + s * a.wstage);
                 // descriptors of the stage's first A row and first B block: an
                 // operand's descriptor is these plus its byte offset / 16 in the
                 // address field (no carry out: shared addresses stay below 256 KB)
-                const uint64_t a0 = umma_desc(stage, 16, 1024, 2), b0 = umma_desc(w_stage, 128, 256, 0);
+                const uint64_t a0 = tc5::desc_sw128(stage), b0 = tc5::desc(w_stage, 128, 256);
                 const uint32_t wb16 = wblock >> 4;
                 int e = lo;
                 if constexpr (!F32 && NISS == 1) {
@@ -315,7 +254,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                         // entries, then issue their MMAs back to back (one
                         // thread issues, so the decoding would otherwise sit
                         // between MMAs)
-                        constexpr uint32_t idesc = idesc_bf16(TN, R);
+                        constexpr uint32_t idesc = tc5::idesc(false, TN, R);
                         for (; e + 4 <= hi; e += 4) {
                             const uint32_t vv[4] = {(uint32_t)ent[e], (uint32_t)ent[e + 1], (uint32_t)ent[e + 2],
                                                     (uint32_t)ent[e + 3]};
@@ -329,7 +268,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                                 acc[jj] = ((vv[jj] >> 7) & 1u) == 0u;
                             }
 #pragma unroll
-                            for (int jj = 0; jj < 4; jj++) mma_bf16(dv[jj], adv[jj], bdv[jj], idesc, acc[jj]);
+                            for (int jj = 0; jj < 4; jj++) tc5::mma_ss<false>(dv[jj], adv[jj], bdv[jj], idesc, acc[jj]);
                         }
                     }
                 }
@@ -345,11 +284,11 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                             // blocks; this issuer's items are rows ufirst*R ..
                             // of it, into their adjacent accumulators
                             const uint32_t ns = (uint32_t)(g_count * R);
-                            const uint32_t idesc_s = idesc_bf16(TN, (int)(ucnt * R));
+                            const uint32_t idesc_s = tc5::idesc(false, TN, (int)(ucnt * R));
                             const uint64_t bs = bd + (uint64_t)(ufirst * R * 2);   // ufirst * R rows of 32 bytes
 #pragma unroll 4
                             for (int sl = 0; sl < C / 16; sl++)
-                                mma_bf16(tmem + ufirst * R, ad + (uint64_t)(sl * 2), bs + (uint64_t)(sl * ns * 2),
+                                tc5::mma_ss<false>(tmem + ufirst * R, ad + (uint64_t)(sl * 2), bs + (uint64_t)(sl * ns * 2),
                                          idesc_s, (first == 0u) | (sl > 0));
                             continue;
                         }
@@ -358,31 +297,31 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                     const uint32_t d = tmem + g * R;
                     if constexpr (F32) {
                         // 3xTF32: high x high + high x low + low x high, K = 8 per MMA
-                        constexpr uint32_t idesc = idesc_tf32(TN, R);
+                        constexpr uint32_t idesc = tc5::idesc(true, TN, R);
                         const uint64_t adl = ad + (uint64_t)(NS * kStageBytes >> 4), bdl = bd + (uint64_t)((uint32_t)R * C * 4 >> 4);
 #pragma unroll 2
                         for (int sl = 0; sl < C / 8; sl++) {
                             const uint64_t ka = (uint64_t)(sl * 2), kb = (uint64_t)(sl * (R * 2));   // 32 and R*32 bytes
-                            mma_tf32(d, ad + ka, bd + kb, idesc, (first == 0u) | (sl > 0));
-                            mma_tf32(d, ad + ka, bdl + kb, idesc, 1u);
-                            mma_tf32(d, adl + ka, bd + kb, idesc, 1u);
+                            tc5::mma_ss<true>(d, ad + ka, bd + kb, idesc, (first == 0u) | (sl > 0));
+                            tc5::mma_ss<true>(d, ad + ka, bdl + kb, idesc, 1u);
+                            tc5::mma_ss<true>(d, adl + ka, bd + kb, idesc, 1u);
                         }
                     } else {
-                        constexpr uint32_t idesc = idesc_bf16(TN, R);
+                        constexpr uint32_t idesc = tc5::idesc(false, TN, R);
 #pragma unroll 4
                         for (int sl = 0; sl < C / 16; sl++)
-                            mma_bf16(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
+                            tc5::mma_ss<false>(d, ad + (uint64_t)(sl * 2), bd + (uint64_t)(sl * (R * 2)), idesc,
                                      (first == 0u) | (sl > 0));
                     }
                 }
-                mma_commit(&empty[s]);   // the stage is free once every issuer's MMAs completed
+                tc5::commit(&empty[s]);   // the stage is free once every issuer's MMAs completed
                 k++;
             }
             if (!ok) {
                 set_status(a.status, DEV_TIMEOUT);
                 atomicExch(&misc[0], 1);
             }
-            mma_commit(done);   // every MMA this issuer issued completes before its `done` arrival
+            tc5::commit(done);   // every MMA this issuer issued completes before its `done` arrival
         }
     } else {
         // ---------------- the last four warps: fp32 split during the main
@@ -428,7 +367,7 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
         // the last commit fires after the whole main loop: allow it every chunk's bound
         const uint64_t limit = a.wait_ns * (uint64_t)(nch + 2);
         const bool got = ptx::mbar_wait_bounded_idle(done, 0, limit);   // the whole main loop: sleep while waiting
-        tc_fence_after();
+        tc5::fence_after();
         const bool stop = ptx::named_barrier_or(1, 128, !got || !split_ok || aborted(misc));
         if (!got && et == 0) set_status(a.status, DEV_TIMEOUT);
         const int q = warp & 3;
@@ -451,9 +390,9 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                 ptx::named_barrier(1, 128);
             }
             uint32_t r0[32], r1[32];
-            tmem_ld32_nowait(lane_base + c0, r0);
-            if (c0 + 32 < g_count * R) tmem_ld32_nowait(lane_base + c0 + 32, r1);
-            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            tc5::ld32(lane_base + c0, r0);
+            if (c0 + 32 < g_count * R) tc5::ld32(lane_base + c0 + 32, r1);
+            tc5::ld_wait();
 #pragma unroll
             for (int h = 0; h < 64; h += 16) {
                 const int col = c0 + h;
@@ -512,11 +451,11 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
     }
     // ---------------- teardown: every MMA completed (the epilogue waited for
     // `done`, or the issuer never started), then free the tensor memory
-    tc_fence_before();
+    tc5::fence_before();
     __syncthreads();
     if (warp == 1) {
-        tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(a.tmem_cols) : "memory");
+        tc5::fence_after();
+        tc5::dealloc(tmem, a.tmem_cols);
     }
 }
 
