@@ -21,8 +21,9 @@
 //                         block is a stack: one MMA per K slice with
 //                         N = items x R over their adjacent accumulators. A
 //                         tcgen05.commit per chunk releases the stage.
-//   warps 2..5           fp32: split every landed X stage into tf32 high and
-//                         low parts (low into a twin buffer) for the issuer's
+//   warps 2..5           fp32: write the tf32 low parts of every landed X
+//                         stage into a twin buffer (the MMAs read the stage
+//                         itself as the high parts) for the issuer's
 //                         high x high + high x low + low x high; then the
 //                         epilogue: each reads its 32 TMEM lanes (tokens),
 //                         adds the bias, converts, stages 16-column groups in
@@ -334,8 +335,12 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
         }
         bool split_ok = true;
         if constexpr (F32) {
-            // x = high + low per element of every loaded stage: high in
-            // place, low into the stage's twin buffer (same swizzled layout)
+            // x = high + low per element of every loaded stage: the low part
+            // into the stage's twin buffer (same swizzled layout); the high
+            // part is the stage itself, since kind::tf32 MMAs use only the
+            // top 19 bits of each fp32 element (round-to-nearest would leave
+            // about 2^-11 relative error per product, far outside the fp32
+            // tolerance the parity tests check)
             split_ok = ptx::mbar_wait_bounded(rbar, 0, a.wait_ns);
             int k = 0;
             for (int c = 0; split_ok && c < nch; c++) {
@@ -350,7 +355,6 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
                     const int q4 = et + 128 * j;
                     const float4 x = hi4[q4];
                     const float4 h = tf32_high(x);
-                    hi4[q4] = h;
                     lo4[q4] = make_float4(x.x - h.x, x.y - h.y, x.z - h.z, x.w - h.w);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the tensor cores
