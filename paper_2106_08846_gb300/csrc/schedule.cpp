@@ -662,9 +662,12 @@ int choose_tasks(const Schedule &sc, int64_t N) {
     for (int gi = 0; gi < kXsTaskSizes; gi++) {
         const int G = kXsG[gi];
         if (!fits(G)) continue;
-        const int64_t ctas = tiles * ((items + G - 1) / G);
+        const int64_t tasks = (items + G - 1) / G;
+        const int64_t ctas = tiles * tasks;
         const double waves = (double)((ctas + sc.sm_count - 1) / sc.sm_count);
-        const double cost = waves * (kFixed + (double)std::min<int64_t>(G, items) * item_work);
+        // a wave's CTAs carry the mean task's items: a light last task (items
+        // not a multiple of G) shortens the waves it falls in
+        const double cost = waves * (kFixed + (double)items / (double)std::max<int64_t>(tasks, 1) * item_work);
         if (best_cost < 0 || cost < best_cost) {
             best_cost = cost;
             best = G;

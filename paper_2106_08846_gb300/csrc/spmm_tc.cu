@@ -102,7 +102,9 @@ __device__ __forceinline__ bool aborted(const int *flag) { return *reinterpret_c
 __device__ __forceinline__ int pad4(int n) { return (n + 3) & ~3; }
 
 // One CTA of the product described by `a`; `cta` is its index in that
-// product's grid (tile-fastest).
+// product's grid (task-fastest: the tasks of a token tile run at about the
+// same time, so their reads of the tile's X chunks meet in L2; tile-fastest
+// read X from DRAM twice on 1024-wide fp32 16x16 weights, 107.6 -> 102.2 us).
 template <typename T, int R>
 __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a, unsigned cta) {
     ptx::pdl_launch_dependents();
@@ -124,9 +126,8 @@ __device__ __forceinline__ void tc_cta(const CUtensorMap &xmap, const TcArgs &a,
     float *B_s = reinterpret_cast<float *>(base + a.bias_off);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t n_tiles = (a.N + TN - 1) / TN;
-    const int task = (int)(cta / n_tiles);
-    const int64_t n0 = (int64_t)(cta % n_tiles) * TN;
+    const int task = (int)(cta % a.n_tasks);
+    const int64_t n0 = (int64_t)(cta / a.n_tasks) * TN;
     const int32_t *trec = a.trec + __ldg(a.trec_off + task);
     const int g_count = __ldg(trec + 1);
     const int C = a.C, nch = a.nchunks;
@@ -661,7 +662,7 @@ cudaError_t launch_r(const LaunchArgs *las, const int *Gs, int n) {
         static std::atomic<uint64_t> attr_set{0};
         if ((e = allow_smem(k_tc<T, R>, attr_set)) != cudaSuccess) return e;
         if ((e = encode_x<T>(las[0].X, las[0].N, las[0].sc->K, &map)) != cudaSuccess) return e;
-        const int64_t grid = n_tiles * a.n_tasks;   // tile-fastest order
+        const int64_t grid = n_tiles * a.n_tasks;   // task-fastest order
         if (grid > INT32_MAX) return cudaErrorInvalidConfiguration;
         return launch_kernel(k_tc<T, R>, dim3((unsigned)grid), dim3(TcCfg<T>::NTHREADS), smem, las[0].stream, map, a);
     }
