@@ -679,6 +679,13 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
         snprintf(gks + at, sizeof gks - at, at ? ",%d" : "%d", kGkG[gi]);
     }
     if (!gks[0]) snprintf(gks, sizeof gks, "none");
+    char xss[64] = "";   // task sizes the SIMT kernel can run (blobs built and within shared memory)
+    for (int gi = 0; gi < kXsTaskSizes && sc.variant == V_XSTAGE; gi++) {
+        if (sc.xs_blob_off[gi] < 0) continue;
+        const size_t at = strlen(xss);
+        snprintf(xss + at, sizeof xss - at, at ? ",%d" : "%d", kXsG[gi]);
+    }
+    if (!xss[0]) snprintf(xss, sizeof xss, "none");
     snprintf(buf, len,
              "variant=%s\ndtype=%s\nR=%d\nC=%d\nexec_R=%d\nexec_C=%d\nM=%" PRId64 "\nK=%" PRId64 "\nMB=%" PRId64
              "\nKB=%" PRId64 "\nnnzb=%" PRId64 "\ntokens_per_cta=%d\nthreads=%d\nsmem_bytes=%zu\n"
@@ -686,12 +693,12 @@ bsr_status_t bsr_get_schedule(bsr_handle_t h, char *buf, size_t len) {
              "empty_rows=%" PRId64 "\nmax_row_blocks=%" PRId64 "\nlaunches_per_call=%d\n"
              "structure_hash=%016" PRIx64 "\ncache_hit=%d\nschedule_reuses=%" PRId64
              "\ncache_hits_total=%" PRId64 "\ncache_misses_total=%" PRId64 "\ntc_stacked_chunks=%s\n"
-             "gk_task_sizes=%s\n",
+             "gk_task_sizes=%s\nxstage_task_sizes=%s\n",
              variant_name(sc.variant), sc.dt == BSR_F32 ? "f32" : "bf16", sc.R, sc.C, sc.ex_R, sc.ex_C, sc.M, sc.K,
              sc.MB, sc.KB, sc.nnzb, sc.tn, sc.threads, sc.smem, sc.groups, sc.items.size(),
              sc.split_len, split_rows, sc.n_slots, sc.empty_rows, sc.max_row, launches_per_call(sc),
              sc.hash, (int)h->cache_hit, (int64_t)sc.reuse_count, (int64_t)g_cache_hits,
-             (int64_t)g_cache_misses, stacks, gks);
+             (int64_t)g_cache_misses, stacks, gks, xss);
     return BSR_OK;
 }
 
