@@ -272,13 +272,15 @@ def test_error_statuses():
     assert h.check_device_status() == b.BSR_OK
 
 
-@pytest.mark.parametrize("R,C,dtype,variant", [(32, 1, "f32", "xstage"), (16, 16, "bf16", "tcgen05"),
-                                               (32, 32, "f32", "tcgen05")])
-def test_bounded_wait_times_out_and_reports(monkeypatch, R, C, dtype, variant):
+@pytest.mark.parametrize("R,C,dtype,variant,N", [(32, 1, "f32", "xstage", 5000), (32, 1, "f32", "xstage", 128),
+                                                 (16, 16, "bf16", "tcgen05", 128), (32, 32, "f32", "tcgen05", 128)])
+def test_bounded_wait_times_out_and_reports(monkeypatch, R, C, dtype, variant, N):
     """An X chunk that is never loaded: every wait on it gives up after the
     bound (2 ms here), the kernel records BSR_ERR_TIMEOUT, releases what it
     holds and returns; the context stays usable and a normal handle still
-    computes correctly."""
+    computes correctly. The SIMT kernel runs once with many token tiles per
+    task (the stalled chunk's waits end in every CTA at once) and once with
+    two."""
     bsr = _bsr()
     from paper_2106_08846_gb300 import bsrlib as b
     w = _weight(256, 512, R, C, dtype, 0.2, 21)
@@ -289,7 +291,7 @@ def test_bounded_wait_times_out_and_reports(monkeypatch, R, C, dtype, variant):
     monkeypatch.delenv("BSR_WAIT_LIMIT_NS")
     monkeypatch.delenv("BSR_TEST_STALL_CHUNK")
     assert h.schedule()["variant"] == variant
-    X = synth.activations(22, 128, 512, dtype)
+    X = synth.activations(22, N, 512, dtype)
     h.spmm(to_dev(X), to_dev(w.bias))
     assert h.check_device_status() == b.BSR_ERR_TIMEOUT
     assert h.check_device_status() == b.BSR_OK          # cleared after reading
