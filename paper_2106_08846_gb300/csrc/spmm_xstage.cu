@@ -2,7 +2,7 @@
 //
 // Each CTA owns a tile of TN = 64 tokens and a task of G work items (block
 // rows or pieces of rows, Section 2.2's kept blocks), with NW consumer warps
-// and one producer warp: S = NW/G warps per item for G <= NW (NW = 12), or,
+// and one producer warp: S = NW/G warps per item for G <= NW (NW = 14), or,
 // for one-row blocks (NW = 24), G/NW whole items per warp when G > NW. The
 // inner product over the kept blocks is FP32-FMA bound, so the design goal
 // is a high share of packed FMAs among the issued instructions:

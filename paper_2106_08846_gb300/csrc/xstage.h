@@ -11,17 +11,22 @@ namespace bsr {
 constexpr int kXsTokens = 64;          // tokens per CTA
 constexpr int kXsChunk = 128;          // K columns per ring stage
 constexpr int kXsStages = 3;           // ring depth
-constexpr int kXsConsumerWarps = 12;   // + 1 producer warp: 16 warps of registers
+constexpr int kXsConsumerWarps = 14;   // + 1 producer warp, up to 136 registers a thread
 constexpr int kXsConsumerWarpsR1 = 24; // one-row blocks (small tiles): + 1 producer warp, 80 registers a thread
 constexpr int kXsMaxSmem = 232448;     // 227 KB, the per-CTA opt-in limit
 constexpr int kXsWDup = 1;             // copies of each packed block value
 constexpr int kXsBatchMax = 64;        // products in one fused launch (bsr_spmm_batch)
 
-// Task sizes G (items per CTA): up to the consumer warps NW, each dividing
-// them (NW/G warps per item); one-row blocks (NW = 24) also G = 48 and 96,
-// two or four items per warp.
-constexpr int kXsTaskSizes = 9;
-constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 12, 24, 48, 96};
+// Task sizes G (items per CTA): up to the consumer warps NW, NW/G (rounded
+// down) warps per item, the rest idle; one-row blocks (NW = 24) take only
+// sizes dividing 24, and also G = 48 and 96, two or four items per warp.
+// Multi-row blocks run fourteen consumer warps: more warps hide more of the
+// multiply-add loop's latency, and fourteen measured faster than twelve even
+// where two of them idle (BERT-large 32x1 fp32: 7-item tasks 139.1 us against
+// 6-item tasks on twelve warps 141.2 us; block-shape sweep 154 against 157
+// us), fifteen slower (146 us: 5-item tasks).
+constexpr int kXsTaskSizes = 11;
+constexpr int kXsG[kXsTaskSizes] = {1, 2, 3, 4, 6, 7, 12, 14, 24, 48, 96};
 
 constexpr int kXsItab = 12;   // ints per item in a task's item table
 

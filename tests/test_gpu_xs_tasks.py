@@ -13,7 +13,7 @@ pytestmark = pytest.mark.gpu
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-@pytest.mark.parametrize("G", ["1", "2", "3", "4", "6", "12", "24", "48", "96"])
+@pytest.mark.parametrize("G", ["1", "2", "3", "4", "6", "7", "12", "14", "24", "48", "96"])
 def test_xs_forced_task_size(G):
     e = dict(os.environ, BSR_XS_G=G, BSR_FORCE_VARIANT="xstage")
     r = subprocess.run([sys.executable, "-m", "tests.xs_task_size_check"], cwd=ROOT, env=e, capture_output=True,

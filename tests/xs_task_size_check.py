@@ -34,7 +34,7 @@ def main() -> int:
     G = int(os.environ["BSR_XS_G"])
     fails = ran = 0
     for R, C, dt, dens, K, N, with_bias in CASES:
-        if G > 12 and R != 1:   # several items per warp: one-row blocks only
+        if G > 14 and R != 1:   # several items per warp: one-row blocks only
             continue
         M = 384
         MB, KB = M // R, K // C
