@@ -25,8 +25,11 @@
  * into a tf32 high part and a tf32 low part (the remainder) and the product is
  * hi*hi + hi*lo + lo*hi, accumulated in fp32. The dropped lo*lo term and the
  * rounding of the low parts leave a relative error near 2^-20 per product,
- * inside the fp32 tolerance |dY| <= 1e-5 * (sum |x||w| + |b|). Every other
- * fp32 shape multiplies in plain fp32 FMA.
+ * inside the fp32 tolerance |dY| <= 1e-5 * (sum |x||w| + |b|). Calls of 512
+ * or more tokens on fp32 blocks that only the generic kernel would take
+ * otherwise (64 or 128 rows with 1 to 8 columns) run on the gathered-K
+ * tensor-core kernel, 3xTF32 in the same way. Every other fp32 shape
+ * multiplies in plain fp32 FMA.
  *
  * Conventions.
  *  - Every call returns a status; the library never aborts, prints or traps.
