@@ -151,8 +151,9 @@ bsr_status_t bsr_check_device_status(bsr_handle_t h);
  * variant, execution block height and width (exec_R x exec_C: max(R, 16) x 64
  * where small or narrow bf16 blocks run on the tensor cores as zero-filled
  * tiles), tile sizes, work items, split
- * rows, launches per call and the schedule-cache statistics, as "key=value"
- * lines. Writes at most len bytes
+ * rows, launches per call, the schedule-cache statistics and the task sizes
+ * each kernel can run (items per CTA; the size a call uses is chosen per
+ * call from its token count), as "key=value" lines. Writes at most len bytes
  * including the terminating NUL into buf (truncating). Returns
  * BSR_ERR_INVALID_ARG for a NULL handle or buffer.
  */
