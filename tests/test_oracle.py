@@ -353,3 +353,60 @@ def test_f32acc_full_sparsity_gives_bias_bf16():
     assert bsr[0][-1] == 0
     Y = oracle.bsr_spmm_f32acc(*bsr, X, b, M, threads=2)
     assert np.array_equal(Y, np.broadcast_to(b, (5, M)))
+
+
+# ---------------------------------------------------------------- property
+
+def _divisors(n):
+    return [d for d in range(1, n + 1) if n % d == 0]
+
+
+def _brute_bsr(W, R, C):
+    """The three arrays written out from Section 2.2's definition, block by
+    block: keep a block iff some element has !(|w| <= 0)."""
+    M, K = W.shape
+    Wf = W.astype(np.float64)
+    indptr, indices, data = [0], [], []
+    for i in range(M // R):
+        for j in range(K // C):
+            blk = Wf[i * R:(i + 1) * R, j * C:(j + 1) * C]
+            if np.any(~(np.abs(blk) <= 0.0)):
+                indices.append(j)
+                data.append(W[i * R:(i + 1) * R, j * C:(j + 1) * C])
+        indptr.append(len(indices))
+    return indptr, indices, data
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_property_random_tiny_shapes_against_brute_force(dtype):
+    """Seeded random cases: M, K <= 64, a block shape (R, C) dividing them,
+    block sparsity from 0% to 100% and 1 to 9 tokens. The builder against the
+    definition written out block by block (indptr, indices, values bit for
+    bit), and the product against explicit sums over the dense weight in
+    float64 -- zeros outside the kept blocks add nothing, and the terms come
+    in the same ascending column order, so the results agree bit for bit."""
+    rng = np.random.default_rng(2106 + (dtype == "bf16"))
+    for case in range(60):
+        M, K = int(rng.integers(1, 65)), int(rng.integers(1, 65))
+        R, C = int(rng.choice(_divisors(M))), int(rng.choice(_divisors(K)))
+        density = float(rng.choice([0.0, 0.15, 0.4, 0.8, 1.0]))
+        W, _ = _block_weight(M, K, R, C, density, 4000 + case, dtype)
+        N = int(rng.integers(1, 10))
+        X = synth.activations(5000 + case, N, K, dtype)
+        b = synth.normal(6000 + case, 0, M, 0.02).astype(np.float32)
+        indptr, indices, data = oracle.bsr_from_dense(W, R, C)
+        e_ptr, e_ind, e_data = _brute_bsr(W, R, C)
+        assert indptr.tolist() == e_ptr and indices.tolist() == e_ind, (case, M, K, R, C)
+        assert data.shape == (len(e_ind), R, C)
+        assert all(np.array_equal(data[p].view(np.uint8), np.ascontiguousarray(e_data[p]).view(np.uint8))
+                   for p in range(len(e_ind)))
+        Y = oracle.bsr_spmm(indptr, indices, data, X, b, M)
+        Wd, Xd = _f64(W), _f64(X)
+        Yb = np.empty((N, M))
+        for n in range(N):
+            for m in range(M):
+                acc = 0.0
+                for k in range(K):
+                    acc += Xd[n, k] * Wd[m, k]
+                Yb[n, m] = acc + float(b[m])
+        assert np.array_equal(Y, Yb), (case, M, K, R, C)
