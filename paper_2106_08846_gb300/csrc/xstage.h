@@ -77,7 +77,7 @@ constexpr int xstage_slot_pitch(int R, int nslot) {
 uint32_t xstage_stage_offset(bsr_dtype_t dt, int kk);
 
 int g_index(int G);
-bool xstage_task_size_ok(int R, int G);   // G > 12 needs one-row blocks
+bool xstage_task_size_ok(int R, int G);   // G > 14 needs one-row blocks
 bool xstage_supports(int R, int C, bsr_dtype_t dt, int64_t K);
 
 // Dynamic shared memory of one CTA: ring (reused for the epilogue's partial
